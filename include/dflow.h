@@ -1,0 +1,201 @@
+/*
+ * dflow.h -- C ABI of the DFlow speculative-decoding round on one GPU.
+ *
+ * One round of block-diffusion speculative decoding with DFlow's verifier
+ * information relay (arXiv 2609.06498):
+ *
+ *   dflow_draft_block   Sec. 3 Eq. 2 with Sec. 4.2 Eq. 4-5: the drafter predicts
+ *                       B future tokens in one forward pass from mask embeddings,
+ *                       relayed verifier states and the fused target context.
+ *   dflow_verify_block  Sec. 3 Eq. 3 (target side) and Eq. 1: one target forward
+ *                       over the anchor and the B proposals against the cached
+ *                       K/V; per-row greedy predictions and fused features.
+ *   dflow_accept_commit Sec. 3 Eq. 3: accepted prefix, bonus token, commit of
+ *                       a+1 tokens, rollback of the rest.
+ *   dflow_carry_hidden  Sec. 3 (context injected into draft K/V) and Sec. 4.2
+ *                       (alignment: keep the shifted verifier states of the
+ *                       rejected suffix and the two boundary tokens).
+ *   dflow_round         the four calls above in order, for the whole batch.
+ *
+ * Conventions shared by every call
+ *   - Pointers in dflow_weights and dflow_state and every output pointer are
+ *     DEVICE pointers, owned by the caller and never freed by the library.
+ *     Structs themselves are read on the host during the call only.
+ *   - The library allocates no device memory after dflow_set_workspace: all
+ *     scratch lives in the caller's workspace.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t passed as void*).
+ *     Argument errors found on the host return a nonzero status synchronously
+ *     and launch nothing.  Errors found on the device (sequence capacity
+ *     exhausted, token id out of range, invalid carried count, a bounded wait
+ *     that timed out) are written to *state->status; every later kernel of the
+ *     library that sees a nonzero status returns without writing.  Read it
+ *     with dflow_read_status.
+ *   - A handle is not thread safe and serves one stream at a time.
+ *   - dtype DFLOW_F32: weights, activations, caches in fp32, fp32 arithmetic.
+ *     dtype DFLOW_BF16: weights, caches, features and carry in bf16; fp32
+ *     accumulation, fp32 residual stream and fp32 norms/softmax/rotary.
+ *
+ * Decoding state invariants (per sequence b, n = seq_len[b] committed tokens)
+ *   tokens[b][0..n-1] committed; tokens[b][n-1] is the anchor.
+ *   Target K/V and drafter context K/V are valid for positions 0..n-2.
+ *   carry slot j (1..n_carry[b]) holds the relayed feature for draft row j.
+ *   Block row i (0..B) of a round sits at position n-1+i.
+ */
+#ifndef DFLOW_H
+#define DFLOW_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum dflow_status {
+  DFLOW_OK = 0,
+  DFLOW_ERR_INVALID_ARG = 1,    /* null pointer, bad size or shape, call order */
+  DFLOW_ERR_CUDA = 2,           /* a CUDA runtime call failed */
+  DFLOW_ERR_CAPACITY = 3,       /* a sequence would grow past max_ctx */
+  DFLOW_ERR_DEVICE_TIMEOUT = 4, /* a bounded device wait gave up */
+  DFLOW_ERR_UNSUPPORTED = 5,    /* shape or device outside what the kernels cover */
+  DFLOW_ERR_BAD_STATE = 6       /* token / count out of range found on the device */
+} dflow_status;
+
+enum { DFLOW_F32 = 0, DFLOW_BF16 = 1 };
+
+#define DFLOW_MAX_FEAT 8
+
+/* Model and workload shape.  head_dim must be 64 or 128, d_model a multiple
+ * of 128, d_inter a multiple of 64.  feat_layers are 1-indexed target layers
+ * (Eq. 1 takes the residual stream after each of them). */
+typedef struct dflow_config {
+  int32_t dtype;
+  int32_t d_model, n_layers, n_q_heads, n_kv_heads, head_dim, d_inter, vocab;
+  int32_t draft_layers, n_feat, feat_layers[DFLOW_MAX_FEAT];
+  int32_t block;     /* B: draft tokens per round; a block has B+1 rows */
+  int32_t page_size; /* tokens per KV page */
+  int32_t max_batch; /* most sequences per call */
+  int32_t max_ctx;   /* token capacity of one sequence (multiple of page_size) */
+  int32_t num_pages; /* pages in each K/V pool */
+  float rope_theta, rms_eps, ln_eps;
+} dflow_config;
+
+/* One decoder layer (Qwen3 layout).  Matrices are row-major [out][in].
+ *   w_qkv     [(Hq + 2 Hkv) * hd][d]: rows of Wq, then Wk, then Wv
+ *   w_o       [d][Hq * hd]
+ *   w_gate_up [2 * d_inter][d]: in groups of 128 rows, rows 0..63 are gate
+ *             rows 64g..64g+63 and rows 64..127 the matching up rows
+ *   w_down    [d][d_inter]
+ * Norm gains are fp32 vectors of d (attn_norm, mlp_norm) or hd (q/k). */
+typedef struct dflow_layer_weights {
+  const void *w_qkv, *w_o, *w_gate_up, *w_down;
+  const float *attn_norm, *mlp_norm, *q_norm, *k_norm;
+} dflow_layer_weights;
+
+/* target: host array of n_layers layers; draft: host array of draft_layers.
+ * embed, lm_head [vocab][d] (LM head shared by target and drafter);
+ * w_c [d][n_feat * d] (Eq. 1); relay_w1 [d][3d], relay_w2 [2d][d] (Eq. 4);
+ * e_mask, ln_w, ln_b, c_norm, final norms: fp32 [d]. */
+typedef struct dflow_weights {
+  const void *embed, *lm_head;
+  const float *final_norm;
+  const dflow_layer_weights *target;
+  const dflow_layer_weights *draft;
+  const float *draft_final_norm;
+  const void *w_c;
+  const float *c_norm;
+  const float *e_mask;
+  const void *relay_w1, *relay_w2;
+  const float *ln_w, *ln_b;
+} dflow_weights;
+
+/* Decoding state of `batch` sequences (device memory).
+ *   tokens     int32 [batch][max_ctx]
+ *   seq_len    int32 [batch]           n
+ *   page_table int32 [batch][max_ctx / page_size]: page id of every logical
+ *              page; fixed for the life of the sequence (commit and rollback
+ *              move only seq_len)
+ *   kv         target pool  [n_layers][num_pages][2][Hkv][page_size][hd]
+ *   draft_kv   drafter pool [draft_layers][num_pages][2][Hkv][page_size][hd]
+ *   carry      [batch][B][d]  (slot j at index j-1)
+ *   n_carry    int32 [batch];  boundary int32 [batch][2] = (bonus, y_{a+1})
+ *   active     int32 [batch]: 0 freezes a sequence (no state writes)
+ *   status     int32 [1]: 0 or a dflow_status written by the device */
+typedef struct dflow_state {
+  int32_t batch;
+  int32_t *tokens, *seq_len;
+  const int32_t *page_table;
+  void *kv, *draft_kv, *carry;
+  int32_t *n_carry, *boundary, *active, *status;
+} dflow_state;
+
+typedef struct dflow_handle dflow_handle;
+
+const char *dflow_status_string(dflow_status s);
+
+/* Validate shapes, copy the weight pointer tables, pick kernels for the
+ * current device.  Allocates host memory only. */
+dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow_handle **out);
+/* Device bytes of scratch the handle needs (activations for max_batch rows,
+ * split-K / split-KV partials, the rotary table). */
+dflow_status dflow_workspace_size(const dflow_handle *h, size_t *bytes);
+/* Hand over scratch (>= dflow_workspace_size bytes, 256-byte aligned).  Fills
+ * constant tables with a synchronous launch on the legacy default stream. */
+dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes);
+dflow_status dflow_destroy(dflow_handle *h);
+
+/* Prompt processing (setup, not part of a round; Sec. 3 committed context):
+ * runs the target over prompt[b][0..len_b-1] (device int32, row stride
+ * prompt_stride), writes target K/V and drafter context for positions
+ * 0..len_b-1, appends the greedy next token as the anchor, sets
+ * seq_len = len_b + 1, n_carry = 0.  prompt_len_host: host int32 [batch]. */
+dflow_status dflow_prefill(dflow_handle *h, dflow_state *st, const int32_t *prompt,
+                           int32_t prompt_stride, const int32_t *prompt_len_host,
+                           void *stream);
+
+/* Sec. 3 Eq. 2 + Sec. 4.2 Eq. 4-5.  block_tokens int32 [batch][B+1]: row 0 =
+ * anchor, rows 1..B = drafter argmax.  Reads tokens, seq_len, drafter
+ * context, carry, n_carry, boundary. */
+dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens,
+                               void *stream);
+
+/* Sec. 3 Eq. 3 (target forward) + Eq. 1.  Reads block_tokens [batch][B+1];
+ * writes target K/V at positions n-1..n-1+B, target_argmax int32
+ * [batch][B+1] (row i = greedy prediction for position n+i), feats
+ * [batch][B+1][d] (Eq. 1, model dtype) and, if logits is non-null, fp32
+ * logits [batch][B+1][vocab]. */
+dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                int32_t *target_argmax, void *feats, float *logits,
+                                void *stream);
+
+/* Sec. 3 Eq. 3.  a = number of leading proposals with block[i] ==
+ * target_argmax[i-1]; if forced_accept (int32 [batch], values 0..B) is
+ * non-null it replaces a.  Commits block[1..a] and bonus target_argmax[a] to
+ * tokens[n..n+a]; seq_len += a+1.  accept_len int32 [batch] (-1 for inactive
+ * sequences); committed int32 [batch][B+1], -1 padded. */
+dflow_status dflow_accept_commit(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                 const int32_t *target_argmax, const int32_t *forced_accept,
+                                 int32_t *accept_len, int32_t *committed, void *stream);
+
+/* Sec. 3 + Sec. 4.2, after dflow_accept_commit of the same round.  Feature
+ * rows 0..a join the drafter context of every draft layer (k = RoPE(k_norm(
+ * W_k f)), v = W_v f at positions n_old-1..n_old-1+a); rows a+1..B-1 become
+ * carry slots 1..B-a-1; boundary = (bonus, block[a+1]) (-1 when a = B). */
+dflow_status dflow_carry_hidden(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                const void *feats, const int32_t *accept_len, void *stream);
+
+/* One full round: draft -> verify -> accept/commit -> carry, with block
+ * tokens, predictions and features in the workspace.  relay = 0 runs the
+ * DFlash baseline (nothing carried, mask embeddings only). */
+dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced_accept,
+                         int32_t *accept_len, int32_t *committed, int32_t relay,
+                         void *stream);
+
+/* Synchronises `stream`, then copies *state->status to *host_status. */
+dflow_status dflow_read_status(dflow_handle *h, const dflow_state *st, int32_t *host_status,
+                               void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DFLOW_H */

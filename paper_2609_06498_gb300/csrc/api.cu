@@ -1,0 +1,918 @@
+// C ABI of the DFlow round: argument checks, workspace layout, the order of
+// kernel launches for each call, and the small fused kernels of the round
+// (embedding gather, norms, rotary/K-V writes, acceptance, carry, relay input).
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
+#include <new>
+#include <vector>
+
+#include "dflow_internal.cuh"
+#include "gemm_tc.cuh"
+
+using namespace dflow;
+
+namespace {
+
+constexpr int PF = 64;  // prompt rows per sequence per prefill step
+
+// ---------------------------------------------------------------------------
+// small kernels
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ float block_sum(float v, float *red) {
+  v = warp_sum(v);
+  const int w = threadIdx.x / 32, l = threadIdx.x % 32, nw = blockDim.x / 32;
+  __syncthreads();
+  if (l == 0) red[w] = v;
+  __syncthreads();
+  float t = l < nw ? red[l] : 0.f;
+  return warp_sum(t);
+}
+
+// rotary table: rope[p][i] = (cos, sin)(p * theta^(-2i/hd)), angles in double
+__global__ void k_rope_table(float2 *rope, int max_ctx, int hd, double theta) {
+  const int half = hd / 2;
+  const long long n = (long long)max_ctx * half;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < n;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int p = (int)(e / half), i = (int)(e % half);
+    const double ang = (double)p * pow(theta, -2.0 * i / hd);
+    double sv, cv;
+    sincos(ang, &sv, &cv);
+    rope[e] = make_float2((float)cv, (float)sv);
+  }
+}
+
+// device-side checks before a round touches the caches
+__global__ void k_guard(const int *tokens, const int *seq_len, const int *n_carry,
+                        const int *boundary, const int *active, int batch, int R, int max_ctx,
+                        int vocab, int B, int *status) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch || !active[b]) return;
+  const int n = seq_len[b];
+  if (n < 1 || n - 1 + R > max_ctx) { set_status(status, DFLOW_ERR_CAPACITY); return; }
+  const int anchor = tokens[(size_t)b * max_ctx + n - 1];
+  const int nc = n_carry[b];
+  if (anchor < 0 || anchor >= vocab || nc < 0 || nc > B - 1) { set_status(status, DFLOW_ERR_BAD_STATE); return; }
+  if (nc > 0) {
+    const int t0 = boundary[2 * b], t1 = boundary[2 * b + 1];
+    if (t0 < 0 || t0 >= vocab || t1 < 0 || t1 >= vocab) set_status(status, DFLOW_ERR_BAD_STATE);
+  }
+}
+
+// rows of a round: row b*R+i at position n_b-1+i; writes allowed for active sequences
+__global__ void k_rows_round(int *pos, int *wr, const int *seq_len, const int *active, int batch,
+                             int R, const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * R) return;
+  const int b = r / R, i = r % R;
+  const bool ok = active[b] != 0;
+  pos[r] = ok ? seq_len[b] - 1 + i : 0;
+  wr[r] = ok;
+}
+
+// rows of prefill step c: row b*PF+i at position c0+i if inside the prompt
+__global__ void k_rows_prefill(int *pos, int *wr, const int *plen, int batch, int c0,
+                               const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * PF) return;
+  const int b = r / PF, p = c0 + r % PF;
+  const bool ok = p < plen[b];
+  pos[r] = ok ? p : 0;
+  wr[r] = ok;
+}
+
+// x[r] = E[tok] (fp32 residual stream); tok = toks[b*stride + i]
+template <typename T>
+__global__ void k_embed(const T *__restrict__ E, const int *__restrict__ toks, int stride, int R,
+                        const int *__restrict__ wr, float *__restrict__ x, int d, int vocab,
+                        int *status) {
+  if (*status) return;
+  const int r = blockIdx.x, b = r / R, i = r % R;
+  int tok = (wr == nullptr || wr[r]) ? toks[(size_t)b * stride + i] : 0;
+  if (tok < 0 || tok >= vocab) {
+    if (threadIdx.x == 0) set_status(status, DFLOW_ERR_BAD_STATE);
+    tok = 0;
+  }
+  for (int c = threadIdx.x; c < d; c += blockDim.x) x[(size_t)r * d + c] = to_f(E[(size_t)tok * d + c]);
+}
+
+// y[r] = x[r] / rms(x[r]) * w   (fp32 in, model dtype out)
+template <typename T>
+__global__ void k_rmsnorm(const float *__restrict__ x, int ldx, const float *__restrict__ w,
+                          T *__restrict__ y, int ldy, int d, float eps, const int *status) {
+  if (*status) return;
+  __shared__ float red[32];
+  const float *xr = x + (size_t)blockIdx.x * ldx;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) ss += xr[c] * xr[c];
+  ss = block_sum(ss, red);
+  const float inv = rsqrtf(ss / d + eps);
+  for (int c = threadIdx.x; c < d; c += blockDim.x)
+    y[(size_t)blockIdx.x * ldy + c] = from_f<T>(xr[c] * inv * w[c]);
+}
+
+// per (row, head): q/k RMSNorm over hd, rotary at pos[r], then write q to
+// q_out, k/v either into a paged pool at pos[r] (when wr[r]) or into block
+// buffers.  The source buffer holds nq query heads, then hkv key heads, then
+// hkv value heads.
+template <typename T, int HD>
+__global__ void __launch_bounds__(128)
+k_qkv_post(Dims D, const float *__restrict__ src, int ld, int nq, const float *__restrict__ qn,
+           const float *__restrict__ kn, const float2 *__restrict__ rope,
+           const int *__restrict__ pos, const int *__restrict__ wr, int R, T *__restrict__ q_out,
+           T *__restrict__ pool, const int *__restrict__ page_table, T *__restrict__ bk,
+           T *__restrict__ bv, const int *status) {
+  if (*status) return;
+  constexpr int J = HD / 32, H2 = HD / 64;
+  const int r = blockIdx.x, lane = threadIdx.x % 32;
+  const int head = blockIdx.y * 4 + threadIdx.x / 32;
+  if (head >= nq + 2 * D.hkv) return;
+  const float *s = src + (size_t)r * ld + (size_t)head * HD;
+  float v[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) v[j] = s[lane + 32 * j];
+  const bool is_q = head < nq, is_k = !is_q && head < nq + D.hkv;
+  if (is_q || is_k) {
+    float ss = 0.f;
+#pragma unroll
+    for (int j = 0; j < J; ++j) ss += v[j] * v[j];
+    ss = warp_sum(ss);
+    const float inv = rsqrtf(ss / HD + D.rms_eps);
+    const float *g = is_q ? qn : kn;
+#pragma unroll
+    for (int j = 0; j < J; ++j) v[j] *= inv * g[lane + 32 * j];
+    const float2 *cs = rope + (size_t)pos[r] * (HD / 2);
+#pragma unroll
+    for (int j = 0; j < H2; ++j) {
+      const float2 t = cs[lane + 32 * j];
+      const float x1 = v[j], x2 = v[j + H2];
+      v[j] = x1 * t.x - x2 * t.y;
+      v[j + H2] = x2 * t.x + x1 * t.y;
+    }
+  }
+  T *dst;
+  if (is_q) {
+    dst = q_out + ((size_t)r * nq + head) * HD;
+  } else {
+    const int kvh = is_k ? head - nq : head - nq - D.hkv;
+    if (bk != nullptr) {
+      dst = (is_k ? bk : bv) + ((size_t)r * D.hkv + kvh) * HD;
+    } else {
+      if (!wr[r]) return;
+      const int b = r / R, p = pos[r];
+      const int page = page_table[(size_t)b * D.pages_per_seq + p / D.page_size];
+      dst = pool + pool_off(D, page, is_k ? 0 : 1, kvh, p % D.page_size);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < J; ++j) dst[lane + 32 * j] = from_f<T>(v[j]);
+}
+
+// stash[r][f*d + c] = x[r][c]: residual stream after a feature layer (Eq. 1 input)
+template <typename T>
+__global__ void k_stash(const float *__restrict__ x, T *__restrict__ stash, int d, int m, int f,
+                        const int *status) {
+  if (*status) return;
+  const size_t r = blockIdx.x;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) stash[r * m * d + (size_t)f * d + c] = from_f<T>(x[r * d + c]);
+}
+
+// g[r] = argmax over the per-tile partials (ties: lowest token id)
+__global__ void k_argmax_reduce(const float *__restrict__ pv, const int *__restrict__ pi, int n_tiles,
+                                int rows, int *__restrict__ g, const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32, lane = threadIdx.x % 32;
+  if (r >= rows) return;
+  float v = -INFINITY;
+  int idx = 0x7fffffff;
+  for (int t = lane; t < n_tiles; t += 32) argmax_merge(v, idx, pv[(size_t)r * n_tiles + t], pi[(size_t)r * n_tiles + t]);
+  warp_argmax(v, idx);
+  if (lane == 0) g[r] = idx;
+}
+
+// relay MLP input (Eq. 4): u = [E(b); E(y_{a+1}); h_j] for each of the B slots
+template <typename T>
+__global__ void k_relay_u(const T *__restrict__ E, const int *__restrict__ boundary,
+                          const T *__restrict__ carry, T *__restrict__ u, int d, int B, int vocab,
+                          const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x, b = r / B, s = r % B;
+  int t0 = boundary[2 * b], t1 = boundary[2 * b + 1];
+  t0 = (t0 < 0 || t0 >= vocab) ? 0 : t0;
+  t1 = (t1 < 0 || t1 >= vocab) ? 0 : t1;
+  T *ur = u + (size_t)r * 3 * d;
+  const T *h = carry + ((size_t)b * B + s) * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    ur[c] = E[(size_t)t0 * d + c];
+    ur[d + c] = E[(size_t)t1 * d + c];
+    ur[2 * d + c] = h[c];
+  }
+}
+
+// drafter inputs (Eq. 5): row 0 = E(anchor); slot j <= n_carry:
+// E_mask + beta * LN(h_j) + gamma; other slots E_mask
+template <typename T>
+__global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__ e_mask,
+                              const int *__restrict__ tokens, const int *__restrict__ seq_len,
+                              int max_ctx, const T *__restrict__ carry, const int *__restrict__ n_carry,
+                              const float *__restrict__ bg, const float *__restrict__ ln_w,
+                              const float *__restrict__ ln_b, float ln_eps, int relay,
+                              float *__restrict__ x, int d, int B, const int *status) {
+  if (*status) return;
+  __shared__ float red[32];
+  const int R = B + 1, r = blockIdx.x, b = r / R, j = r % R;
+  float *xr = x + (size_t)r * d;
+  if (j == 0) {
+    const int tok = tokens[(size_t)b * max_ctx + seq_len[b] - 1];
+    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = to_f(E[(size_t)tok * d + c]);
+    return;
+  }
+  if (!relay || j > n_carry[b]) {
+    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = e_mask[c];
+    return;
+  }
+  const T *h = carry + ((size_t)b * B + j - 1) * d;
+  float s1 = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) s1 += to_f(h[c]);
+  const float mu = block_sum(s1, red) / d;
+  float s2 = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const float t = to_f(h[c]) - mu;
+    s2 += t * t;
+  }
+  const float inv = rsqrtf(block_sum(s2, red) / d + ln_eps);
+  const float *beta = bg + ((size_t)b * B + j - 1) * 2 * d, *gamma = beta + d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const float ln = (to_f(h[c]) - mu) * inv * ln_w[c] + ln_b[c];
+    xr[c] = e_mask[c] + beta[c] * ln + gamma[c];
+  }
+}
+
+__global__ void k_draft_out(const int *__restrict__ gd, const int *__restrict__ tokens,
+                            const int *__restrict__ seq_len, int max_ctx, int batch, int R,
+                            int *__restrict__ blk, const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * R) return;
+  const int b = r / R, i = r % R;
+  blk[r] = i == 0 ? tokens[(size_t)b * max_ctx + seq_len[b] - 1] : gd[r];
+}
+
+// Eq. 3: a, bonus, commit (one thread per sequence)
+__global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
+                         const int *__restrict__ forced, int *__restrict__ tokens,
+                         int *__restrict__ seq_len, const int *__restrict__ active, int batch, int B,
+                         int max_ctx, int *__restrict__ acc, int *__restrict__ comm, int *status) {
+  if (*status) return;
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  const int R = B + 1;
+  const int *bb = blk + (size_t)b * R, *gb = g + (size_t)b * R;
+  int *cb = comm + (size_t)b * R;
+  if (!active[b]) {
+    acc[b] = -1;
+    for (int i = 0; i < R; ++i) cb[i] = -1;
+    return;
+  }
+  int a = 0;
+  while (a < B && bb[a + 1] == gb[a]) ++a;
+  if (forced != nullptr) {
+    const int f = forced[b];
+    if (f < 0 || f > B) { set_status(status, DFLOW_ERR_BAD_STATE); return; }
+    a = f;
+  }
+  const int n = seq_len[b];
+  if (n + a + 1 > max_ctx) { set_status(status, DFLOW_ERR_CAPACITY); return; }
+  for (int i = 0; i < R; ++i) {
+    const int t = i < a ? bb[i + 1] : (i == a ? gb[a] : -1);
+    cb[i] = t;
+    if (i <= a) tokens[(size_t)b * max_ctx + n + i] = t;
+  }
+  seq_len[b] = n + a + 1;
+  acc[b] = a;
+}
+
+// positions of the rows that join the drafter context after a commit
+__global__ void k_carry_rows(const int *__restrict__ acc, const int *__restrict__ seq_len, int batch,
+                             int R, int *__restrict__ pos, int *__restrict__ wr, const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * R) return;
+  const int b = r / R, i = r % R, a = acc[b];
+  const bool ok = a >= 0 && i <= a;
+  pos[r] = ok ? seq_len[b] - a - 2 + i : 0;
+  wr[r] = ok;
+}
+
+// Sec. 4.2 alignment: slot j = s+1 <- feature row a+j, for j <= B-a-1
+template <typename T>
+__global__ void k_carry(const T *__restrict__ feats, const int *__restrict__ acc,
+                        const int *__restrict__ blk, const int *__restrict__ tokens,
+                        const int *__restrict__ seq_len, int max_ctx, T *__restrict__ carry,
+                        int *__restrict__ n_carry, int *__restrict__ boundary, int d, int B,
+                        int relay, const int *status) {
+  if (*status) return;
+  const int b = blockIdx.x, s = blockIdx.y, R = B + 1, a = acc[b];
+  if (a < 0) return;
+  const int nc = relay ? max(0, B - a - 1) : 0;
+  if (s == 0 && threadIdx.x == 0) {
+    n_carry[b] = nc;
+    boundary[2 * b] = tokens[(size_t)b * max_ctx + seq_len[b] - 1];
+    boundary[2 * b + 1] = a < B ? blk[(size_t)b * R + a + 1] : -1;
+  }
+  if (s >= nc) return;
+  const T *src = feats + ((size_t)b * R + a + 1 + s) * d;
+  T *dst = carry + ((size_t)b * B + s) * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) dst[c] = src[c];
+}
+
+// prefill bookkeeping for step c: commit prompt tokens, anchor = argmax at len-1
+__global__ void k_prefill_commit(const int *__restrict__ prompt, int stride,
+                                 const int *__restrict__ plen, const int *__restrict__ pos,
+                                 const int *__restrict__ wr, const int *__restrict__ g, int batch,
+                                 int max_ctx, int *__restrict__ tokens, int *__restrict__ seq_len,
+                                 int *__restrict__ n_carry, int *__restrict__ boundary,
+                                 const int *status) {
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * PF || !wr[r]) return;
+  const int b = r / PF, p = pos[r], len = plen[b];
+  tokens[(size_t)b * max_ctx + p] = prompt[(size_t)b * stride + p];
+  if (p == len - 1) {
+    tokens[(size_t)b * max_ctx + len] = g[r];
+    seq_len[b] = len + 1;
+    n_carry[b] = 0;
+    boundary[2 * b] = -1;
+    boundary[2 * b + 1] = -1;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host helpers
+// ---------------------------------------------------------------------------
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace
+
+struct dflow_handle {
+  dflow_config cfg;
+  dflow_weights w;
+  std::vector<dflow_layer_weights> tl, dl;
+  Dims D;
+  int dtype, esz, R, rows_round, rows_max, vocab_tiles, sm_count, gld;
+  int attn_split_round, attn_split_pf;
+  size_t attn_entries;
+  bool use_tc;
+  size_t ws_need = 0, ws_bytes = 0;
+  char *ws = nullptr;
+  // workspace views
+  float *x, *gf32, *apart, *am_val;
+  float2 *rope;
+  void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
+  int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen;
+  TcWorkspace tcw;
+};
+
+namespace {
+
+#define CK(expr)                                     \
+  do {                                               \
+    cudaError_t e_ = (expr);                         \
+    if (e_ != cudaSuccess) return DFLOW_ERR_CUDA;    \
+  } while (0)
+
+struct Call {
+  dflow_handle *h;
+  const int *status;
+  int *status_w;
+  cudaStream_t s;
+};
+
+size_t layout(dflow_handle *h, char *base) {
+  const dflow_config &c = h->cfg;
+  const Dims &D = h->D;
+  size_t off = 0;
+  auto take = [&](size_t bytes) -> char * {
+    char *p = base ? base + off : nullptr;
+    off += align256(bytes);
+    return p;
+  };
+  const size_t rm = h->rows_max, es = h->esz;
+  const int qd = D.hq * D.hd, kvd = D.hkv * D.hd;
+  h->x = (float *)take(rm * D.d * 4);
+  h->gf32 = (float *)take(rm * h->gld * 4);
+  h->xn = take(rm * D.d * es);
+  h->q = take(rm * qd * es);
+  h->bk = take(rm * kvd * es);
+  h->bv = take(rm * kvd * es);
+  h->ao = take(rm * qd * es);
+  h->mlp = take(rm * D.inter * es);
+  h->stash = take(rm * (size_t)D.n_feat * D.d * es);
+  h->feats = take(rm * D.d * es);
+  h->relay_u = take((size_t)c.max_batch * D.B * 3 * D.d * es);
+  h->relay_h = take((size_t)c.max_batch * D.B * D.d * es);
+  h->apart = (float *)take(h->attn_entries * (D.hd + 2) * 4);
+  h->am_val = (float *)take(rm * h->vocab_tiles * 4);
+  h->am_idx = (int *)take(rm * h->vocab_tiles * 4);
+  h->pos = (int *)take(rm * 4);
+  h->wr = (int *)take(rm * 4);
+  h->pos2 = (int *)take(rm * 4);
+  h->wr2 = (int *)take(rm * 4);
+  h->blk = (int *)take(rm * 4);
+  h->g = (int *)take(rm * 4);
+  h->gd = (int *)take(rm * 4);
+  h->acc = (int *)take((size_t)c.max_batch * 4);
+  h->comm = (int *)take(rm * 4);
+  h->plen = (int *)take((size_t)c.max_batch * 4);
+  h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
+  tc_layout(h->tcw, base, off, h->sm_count, rm);
+  return off;
+}
+
+int pick_splits(const dflow_handle *h, int batch, int rows) {
+  int want = (2 * h->sm_count + h->D.hkv * batch - 1) / (h->D.hkv * batch);
+  const int cap = (int)(h->attn_entries / ((size_t)rows * h->D.hq));
+  return std::max(1, std::min(std::min(want, cap), 64));
+}
+
+cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int M, int ldx,
+                 const EpArgs &ep) {
+  dflow_handle *h = k.h;
+  if (h->use_tc && tc_supports(N, K, M, ldx, ep)) return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s);
+  return gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, k.status, k.s);
+}
+
+EpArgs ep_f32(float *out, int ldo, int mode = EP_STORE_F32) {
+  EpArgs e{};
+  e.mode = mode;
+  e.out_f32 = out;
+  e.ldo = ldo;
+  return e;
+}
+EpArgs ep_t(int mode, void *out, int ldt) {
+  EpArgs e{};
+  e.mode = mode;
+  e.out_t = out;
+  e.ldt = ldt;
+  return e;
+}
+
+template <typename T>
+cudaError_t rmsnorm(const Call &k, const float *x, int ldx, const float *w, void *y, int ldy, int rows) {
+  const Dims &D = k.h->D;
+  k_rmsnorm<T><<<rows, 256, 0, k.s>>>(x, ldx, w, static_cast<T *>(y), ldy, D.d, D.rms_eps, k.status);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t qkv_post(const Call &k, const Dims &D, int rows, const float *src, int ld, int nq,
+                     const float *qn, const float *kn, const int *pos, const int *wr, void *q_out,
+                     void *pool, const int *pt, void *bk, void *bv) {
+  const int heads = nq + 2 * D.hkv;
+  dim3 grid(rows, (heads + 3) / 4);
+  if (D.hd == 128)
+    k_qkv_post<T, 128><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+                                               (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status);
+  else
+    k_qkv_post<T, 64><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+                                              (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status);
+  return cudaGetLastError();
+}
+
+// One Qwen3 decoder layer over `rows` rows held in h->x (fp32 residual).
+//   causal = 1: target layer; K/V written to the paged pool (rows with wr),
+//               attention over positions 0..pos.
+//   causal = 0: drafter layer; block K/V kept in bk/bv, attention over the
+//               drafter context pool (0..n-2) and the block rows.
+template <typename T>
+cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_layer_weights &L,
+                          void *pool_layer, const dflow_state *st, int causal, int splits) {
+  dflow_handle *h = k.h;
+  const int rows = batch * D.R, qkv_dim = (D.hq + 2 * D.hkv) * D.hd, qd = D.hq * D.hd;
+  cudaError_t e;
+  if ((e = rmsnorm<T>(k, h->x, D.d, L.attn_norm, h->xn, D.d, rows))) return e;
+  if ((e = gemm(k, L.w_qkv, qkv_dim, D.d, h->xn, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
+  if ((e = qkv_post<T>(k, D, rows, h->gf32, h->gld, D.hq, L.q_norm, L.k_norm, h->pos, h->wr, h->q,
+                       causal ? pool_layer : nullptr, st->page_table, causal ? nullptr : h->bk,
+                       causal ? nullptr : h->bv)))
+    return e;
+  AttnArgs a{};
+  a.q = h->q;
+  a.pool = pool_layer;
+  a.page_table = st->page_table;
+  a.bk = causal ? nullptr : h->bk;
+  a.bv = causal ? nullptr : h->bv;
+  a.pos = h->pos;
+  a.seq_len = st->seq_len;
+  a.causal = causal;
+  a.n_splits = splits;
+  a.part = h->apart;
+  a.out = h->ao;
+  if ((e = attention(h->dtype, D, batch, a, k.status, k.s))) return e;
+  if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, ep_f32(h->x, D.d, EP_RESID)))) return e;
+  if ((e = rmsnorm<T>(k, h->x, D.d, L.mlp_norm, h->xn, D.d, rows))) return e;
+  if ((e = gemm(k, L.w_gate_up, 2 * D.inter, D.d, h->xn, rows, D.d, ep_t(EP_SWIGLU, h->mlp, D.inter)))) return e;
+  return gemm(k, L.w_down, D.d, D.inter, h->mlp, rows, D.inter, ep_f32(h->x, D.d, EP_RESID));
+}
+
+// final RMSNorm -> LM head -> greedy token per row (and fp32 logits when asked)
+template <typename T>
+cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *norm, int *g,
+                           float *logits) {
+  dflow_handle *h = k.h;
+  cudaError_t e;
+  if ((e = rmsnorm<T>(k, h->x, D.d, norm, h->xn, D.d, rows))) return e;
+  EpArgs ep{};
+  ep.mode = EP_ARGMAX;
+  ep.part_val = h->am_val;
+  ep.part_idx = h->am_idx;
+  ep.n_tiles = h->vocab_tiles;
+  if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
+  k_argmax_reduce<<<(rows + 7) / 8, 256, 0, k.s>>>(h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status);
+  if ((e = cudaGetLastError())) return e;
+  if (logits) return gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep_f32(logits, D.vocab));
+  return cudaSuccess;
+}
+
+// target forward over h->x (embeddings) at h->pos; writes K/V, g, Eq. 1 features
+template <typename T>
+cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_state *st, int *g,
+                           void *feats, float *logits, int splits) {
+  dflow_handle *h = k.h;
+  const int rows = batch * D.R;
+  cudaError_t e;
+  int f = 0;
+  for (int l = 0; l < h->cfg.n_layers; ++l) {
+    T *pool_l = static_cast<T *>(st->kv) + (size_t)l * pool_layer_elems(D);
+    if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits))) return e;
+    for (int fi = 0; fi < D.n_feat; ++fi) {
+      if (h->cfg.feat_layers[fi] == l + 1) {
+        k_stash<T><<<rows, 256, 0, k.s>>>(h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status);
+        if ((e = cudaGetLastError())) return e;
+        ++f;
+      }
+    }
+  }
+  if ((e = lm_head_argmax<T>(k, D, rows, h->w.final_norm, g, logits))) return e;
+  // Eq. 1: H_T = RMSNorm(W_c [H^l1; ...; H^lm])
+  if ((e = gemm(k, h->w.w_c, D.d, D.n_feat * D.d, h->stash, rows, D.n_feat * D.d, ep_f32(h->gf32, h->gld)))) return e;
+  return rmsnorm<T>(k, h->gf32, h->gld, h->w.c_norm, feats, D.d, rows);
+}
+
+// drafter context injection: K/V of feature rows (wr2) at pos2 in every draft layer
+template <typename T>
+cudaError_t ctx_append(const Call &k, const Dims &D, int rows, const dflow_state *st, const void *feats) {
+  dflow_handle *h = k.h;
+  cudaError_t e;
+  const size_t qoff = (size_t)D.hq * D.hd * D.d;  // K and V rows follow the Q rows of w_qkv
+  for (int l = 0; l < h->cfg.draft_layers; ++l) {
+    const dflow_layer_weights &L = h->dl[l];
+    const T *wkv = static_cast<const T *>(L.w_qkv) + qoff;
+    if ((e = gemm(k, wkv, 2 * D.hkv * D.hd, D.d, feats, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
+    T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
+    if ((e = qkv_post<T>(k, D, rows, h->gf32, h->gld, 0, nullptr, L.k_norm, h->pos2, h->wr2, nullptr,
+                         pool_l, st->page_table, nullptr, nullptr)))
+      return e;
+  }
+  return cudaSuccess;
+}
+
+Dims round_dims(const dflow_handle *h) {
+  Dims D = h->D;
+  D.R = h->R;
+  return D;
+}
+
+template <typename T>
+dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
+  dflow_handle *h = k.h;
+  const Dims D = round_dims(h);
+  const int batch = st->batch, rows = batch * D.R, B = D.B;
+  k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status);
+  CK(cudaGetLastError());
+  if (relay) {
+    // Eq. 4 for every slot of every sequence; Eq. 5 keeps slots j <= n_carry
+    k_relay_u<T><<<batch * B, 256, 0, k.s>>>((const T *)h->w.embed, st->boundary, (const T *)st->carry,
+                                             (T *)h->relay_u, D.d, B, D.vocab, k.status);
+    CK(cudaGetLastError());
+    CK(gemm(k, h->w.relay_w1, D.d, 3 * D.d, h->relay_u, batch * B, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)));
+    CK(gemm(k, h->w.relay_w2, 2 * D.d, D.d, h->relay_h, batch * B, D.d, ep_f32(h->gf32, 2 * D.d)));
+  }
+  k_draft_input<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
+                                          h->cfg.max_ctx, (const T *)st->carry, st->n_carry, h->gf32,
+                                          h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B, k.status);
+  CK(cudaGetLastError());
+  const int splits = pick_splits(h, batch, rows);
+  for (int l = 0; l < h->cfg.draft_layers; ++l) {
+    T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
+    CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits));
+  }
+  CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
+  k_draft_out<<<(rows + 127) / 128, 128, 0, k.s>>>(h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
+                                                   D.R, blk, k.status);
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
+template <typename T>
+dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, void *feats, float *logits) {
+  dflow_handle *h = k.h;
+  const Dims D = round_dims(h);
+  const int batch = st->batch, rows = batch * D.R;
+  k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status);
+  CK(cudaGetLastError());
+  k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w);
+  CK(cudaGetLastError());
+  CK(target_forward<T>(k, D, batch, st, g, feats, logits, pick_splits(h, batch, rows)));
+  return DFLOW_OK;
+}
+
+dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
+                       int *acc, int *comm) {
+  dflow_handle *h = k.h;
+  k_accept<<<(st->batch + 31) / 32, 32, 0, k.s>>>(blk, g, forced, st->tokens, st->seq_len, st->active,
+                                                 st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w);
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
+template <typename T>
+dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void *feats, const int *acc,
+                      int relay) {
+  dflow_handle *h = k.h;
+  const Dims D = round_dims(h);
+  const int batch = st->batch, rows = batch * D.R;
+  k_carry_rows<<<(rows + 127) / 128, 128, 0, k.s>>>(acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status);
+  CK(cudaGetLastError());
+  CK(ctx_append<T>(k, D, rows, st, feats));
+  k_carry<T><<<dim3(batch, D.B), 256, 0, k.s>>>((const T *)feats, acc, blk, st->tokens, st->seq_len,
+                                               h->cfg.max_ctx, (T *)st->carry, st->n_carry, st->boundary,
+                                               D.d, D.B, relay, k.status);
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
+dflow_status guard(const Call &k, dflow_state *st) {
+  dflow_handle *h = k.h;
+  k_guard<<<(st->batch + 127) / 128, 128, 0, k.s>>>(st->tokens, st->seq_len, st->n_carry, st->boundary,
+                                                   st->active, st->batch, h->R, h->cfg.max_ctx,
+                                                   h->D.vocab, h->D.B, k.status_w);
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
+template <typename T>
+dflow_status do_prefill(const Call &k, dflow_state *st, const int *prompt, int stride, const int *plen_host) {
+  dflow_handle *h = k.h;
+  Dims D = h->D;
+  D.R = PF;
+  const int batch = st->batch, rows = batch * PF;
+  int maxlen = 0;
+  for (int b = 0; b < batch; ++b) maxlen = std::max(maxlen, plen_host[b]);
+  CK(cudaMemcpyAsync(h->plen, plen_host, sizeof(int) * batch, cudaMemcpyHostToDevice, k.s));
+  const int splits = pick_splits(h, batch, rows);
+  for (int c0 = 0; c0 < maxlen; c0 += PF) {
+    k_rows_prefill<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, h->plen, batch, c0, k.status);
+    CK(cudaGetLastError());
+    k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
+                                      D.vocab, k.status_w);
+    CK(cudaGetLastError());
+    CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, splits));
+    k_prefill_commit<<<(rows + 127) / 128, 128, 0, k.s>>>(prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
+                                                          h->cfg.max_ctx, st->tokens, st->seq_len,
+                                                          st->n_carry, st->boundary, k.status);
+    CK(cudaGetLastError());
+    CK(cudaMemcpyAsync(h->pos2, h->pos, sizeof(int) * rows, cudaMemcpyDeviceToDevice, k.s));
+    CK(cudaMemcpyAsync(h->wr2, h->wr, sizeof(int) * rows, cudaMemcpyDeviceToDevice, k.s));
+    CK(ctx_append<T>(k, D, rows, st, h->feats));
+  }
+  return DFLOW_OK;
+}
+
+dflow_status check_call(dflow_handle *h, const dflow_state *st) {
+  if (!h || !st) return DFLOW_ERR_INVALID_ARG;
+  if (!h->ws) return DFLOW_ERR_INVALID_ARG;
+  if (st->batch < 1 || st->batch > h->cfg.max_batch) return DFLOW_ERR_INVALID_ARG;
+  if (!st->tokens || !st->seq_len || !st->page_table || !st->kv || !st->draft_kv || !st->carry ||
+      !st->n_carry || !st->boundary || !st->active || !st->status)
+    return DFLOW_ERR_INVALID_ARG;
+  return DFLOW_OK;
+}
+
+Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
+  return Call{h, st->status, st->status, (cudaStream_t)stream};
+}
+
+bool valid_layer(const dflow_layer_weights &L) {
+  return L.w_qkv && L.w_o && L.w_gate_up && L.w_down && L.attn_norm && L.mlp_norm && L.q_norm && L.k_norm;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+extern "C" {
+
+const char *dflow_status_string(dflow_status s) {
+  switch (s) {
+    case DFLOW_OK: return "ok";
+    case DFLOW_ERR_INVALID_ARG: return "invalid argument";
+    case DFLOW_ERR_CUDA: return "CUDA runtime error";
+    case DFLOW_ERR_CAPACITY: return "sequence capacity exhausted";
+    case DFLOW_ERR_DEVICE_TIMEOUT: return "bounded device wait timed out";
+    case DFLOW_ERR_UNSUPPORTED: return "unsupported shape or device";
+    case DFLOW_ERR_BAD_STATE: return "token or count out of range";
+  }
+  return "unknown status";
+}
+
+dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow_handle **out) {
+  if (!cfg || !w || !out) return DFLOW_ERR_INVALID_ARG;
+  *out = nullptr;
+  const dflow_config &c = *cfg;
+  if (c.dtype != DFLOW_F32 && c.dtype != DFLOW_BF16) return DFLOW_ERR_INVALID_ARG;
+  if (c.d_model <= 0 || c.n_layers <= 0 || c.n_q_heads <= 0 || c.n_kv_heads <= 0 || c.d_inter <= 0 ||
+      c.vocab <= 0 || c.draft_layers <= 0 || c.block <= 0 || c.page_size <= 0 || c.max_batch <= 0 ||
+      c.max_ctx <= 0 || c.num_pages <= 0)
+    return DFLOW_ERR_INVALID_ARG;
+  if (c.head_dim != 64 && c.head_dim != 128) return DFLOW_ERR_UNSUPPORTED;
+  if (c.d_model % 128 || c.d_inter % 64 || c.n_q_heads % c.n_kv_heads || c.max_ctx % c.page_size)
+    return DFLOW_ERR_UNSUPPORTED;
+  if (c.n_feat < 1 || c.n_feat > DFLOW_MAX_FEAT) return DFLOW_ERR_INVALID_ARG;
+  for (int i = 0; i < c.n_feat; ++i)
+    if (c.feat_layers[i] < 1 || c.feat_layers[i] > c.n_layers) return DFLOW_ERR_INVALID_ARG;
+  if (!w->embed || !w->lm_head || !w->final_norm || !w->target || !w->draft || !w->draft_final_norm ||
+      !w->w_c || !w->c_norm || !w->e_mask || !w->relay_w1 || !w->relay_w2 || !w->ln_w || !w->ln_b)
+    return DFLOW_ERR_INVALID_ARG;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!valid_layer(w->target[l])) return DFLOW_ERR_INVALID_ARG;
+  for (int l = 0; l < c.draft_layers; ++l)
+    if (!valid_layer(w->draft[l])) return DFLOW_ERR_INVALID_ARG;
+
+  dflow_handle *h = new (std::nothrow) dflow_handle();
+  if (!h) return DFLOW_ERR_INVALID_ARG;
+  h->cfg = c;
+  h->w = *w;
+  h->tl.assign(w->target, w->target + c.n_layers);
+  h->dl.assign(w->draft, w->draft + c.draft_layers);
+  h->w.target = h->tl.data();
+  h->w.draft = h->dl.data();
+  Dims &D = h->D;
+  D.d = c.d_model;
+  D.hq = c.n_q_heads;
+  D.hkv = c.n_kv_heads;
+  D.hd = c.head_dim;
+  D.inter = c.d_inter;
+  D.vocab = c.vocab;
+  D.B = c.block;
+  D.R = c.block + 1;
+  D.page_size = c.page_size;
+  D.num_pages = c.num_pages;
+  D.max_ctx = c.max_ctx;
+  D.pages_per_seq = c.max_ctx / c.page_size;
+  D.n_feat = c.n_feat;
+  D.rms_eps = c.rms_eps;
+  D.ln_eps = c.ln_eps;
+  h->dtype = c.dtype;
+  h->esz = c.dtype == DFLOW_BF16 ? 2 : 4;
+  h->R = c.block + 1;
+  h->rows_round = c.max_batch * h->R;
+  h->rows_max = c.max_batch * std::max(h->R, PF);
+  h->vocab_tiles = (c.vocab + 127) / 128;
+  h->gld = std::max((c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim, 2 * c.d_model);
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaGetLastError();
+  h->sm_count = sms > 0 ? sms : 148;
+  const int sr = std::min(64, std::max(1, (2 * h->sm_count + c.n_kv_heads * c.max_batch - 1) / (c.n_kv_heads * c.max_batch)));
+  h->attn_entries = std::max((size_t)h->rows_round * c.n_q_heads * sr, (size_t)h->rows_max * c.n_q_heads * std::min(sr, 4));
+  h->use_tc = false;
+  if (c.dtype == DFLOW_BF16) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess)
+      h->use_tc = (major == 10 && minor == 3) && getenv("DFLOW_DISABLE_TC") == nullptr;
+    cudaGetLastError();
+  }
+  h->ws_need = layout(h, nullptr);
+  *out = h;
+  return DFLOW_OK;
+}
+
+dflow_status dflow_workspace_size(const dflow_handle *h, size_t *bytes) {
+  if (!h || !bytes) return DFLOW_ERR_INVALID_ARG;
+  *bytes = h->ws_need;
+  return DFLOW_OK;
+}
+
+dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes) {
+  if (!h || !dev || bytes < h->ws_need || ((uintptr_t)dev & 255)) return DFLOW_ERR_INVALID_ARG;
+  h->ws = static_cast<char *>(dev);
+  h->ws_bytes = bytes;
+  layout(h, h->ws);
+  const long long n = (long long)h->cfg.max_ctx * (h->D.hd / 2);
+  k_rope_table<<<(int)std::min<long long>((n + 255) / 256, 4096), 256>>>(h->rope, h->cfg.max_ctx, h->D.hd,
+                                                                          (double)h->cfg.rope_theta);
+  CK(cudaGetLastError());
+  if (h->use_tc) CK(tc_init(h->tcw, 0));
+  CK(cudaDeviceSynchronize());
+  return DFLOW_OK;
+}
+
+dflow_status dflow_destroy(dflow_handle *h) {
+  if (!h) return DFLOW_ERR_INVALID_ARG;
+  delete h;
+  return DFLOW_OK;
+}
+
+dflow_status dflow_prefill(dflow_handle *h, dflow_state *st, const int32_t *prompt, int32_t prompt_stride,
+                           const int32_t *prompt_len_host, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!prompt || !prompt_len_host || prompt_stride < 1) return DFLOW_ERR_INVALID_ARG;
+  for (int b = 0; b < st->batch; ++b) {
+    const int len = prompt_len_host[b];
+    if (len < 1 || len > prompt_stride) return DFLOW_ERR_INVALID_ARG;
+    if (len + 1 + h->R > h->cfg.max_ctx) return DFLOW_ERR_CAPACITY;
+  }
+  Call k = make_call(h, st, stream);
+  return h->dtype == DFLOW_BF16 ? do_prefill<bf16>(k, st, prompt, prompt_stride, prompt_len_host)
+                                : do_prefill<float>(k, st, prompt, prompt_stride, prompt_len_host);
+}
+
+dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!block_tokens) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  if ((r = guard(k, st))) return r;
+  return h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1) : do_draft<float>(k, st, block_tokens, 1);
+}
+
+dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                int32_t *target_argmax, void *feats, float *logits, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!block_tokens || !target_argmax || !feats) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  if ((r = guard(k, st))) return r;
+  return h->dtype == DFLOW_BF16 ? do_verify<bf16>(k, st, block_tokens, target_argmax, feats, logits)
+                                : do_verify<float>(k, st, block_tokens, target_argmax, feats, logits);
+}
+
+dflow_status dflow_accept_commit(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                 const int32_t *target_argmax, const int32_t *forced_accept,
+                                 int32_t *accept_len, int32_t *committed, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!block_tokens || !target_argmax || !accept_len || !committed) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  return do_accept(k, st, block_tokens, target_argmax, forced_accept, accept_len, committed);
+}
+
+dflow_status dflow_carry_hidden(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
+                                const void *feats, const int32_t *accept_len, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!block_tokens || !feats || !accept_len) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  return h->dtype == DFLOW_BF16 ? do_carry<bf16>(k, st, block_tokens, feats, accept_len, 1)
+                                : do_carry<float>(k, st, block_tokens, feats, accept_len, 1);
+}
+
+dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced_accept, int32_t *accept_len,
+                         int32_t *committed, int32_t relay, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!accept_len || !committed) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  if ((r = guard(k, st))) return r;
+  if (h->dtype == DFLOW_BF16) {
+    if ((r = do_draft<bf16>(k, st, h->blk, relay))) return r;
+    if ((r = do_verify<bf16>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
+    if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return r;
+    return do_carry<bf16>(k, st, h->blk, h->feats, accept_len, relay);
+  }
+  if ((r = do_draft<float>(k, st, h->blk, relay))) return r;
+  if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
+  if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return r;
+  return do_carry<float>(k, st, h->blk, h->feats, accept_len, relay);
+}
+
+dflow_status dflow_read_status(dflow_handle *h, const dflow_state *st, int32_t *host_status, void *stream) {
+  if (!h || !st || !st->status || !host_status) return DFLOW_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize((cudaStream_t)stream));
+  CK(cudaMemcpy(host_status, st->status, sizeof(int32_t), cudaMemcpyDeviceToHost));
+  return DFLOW_OK;
+}
+
+}  // extern "C"

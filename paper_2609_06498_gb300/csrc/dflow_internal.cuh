@@ -1,0 +1,111 @@
+// Internal declarations shared by the translation units of libdflow.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dflow.h"
+
+namespace dflow {
+
+typedef __nv_bfloat16 bf16;
+
+// ---------------------------------------------------------------------------
+// element conversions
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+// (value, index) max with ties to the lowest index
+__device__ __forceinline__ void argmax_merge(float &v, int &i, float v2, int i2) {
+  if (v2 > v || (v2 == v && i2 < i)) { v = v2; i = i2; }
+}
+__device__ __forceinline__ void warp_argmax(float &v, int &i) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    float v2 = __shfl_xor_sync(0xffffffffu, v, o);
+    int i2 = __shfl_xor_sync(0xffffffffu, i, o);
+    argmax_merge(v, i, v2, i2);
+  }
+}
+
+// first device-detected error wins
+__device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, 0, code); }
+
+// ---------------------------------------------------------------------------
+// GEMM: out[m][n] = sum_k X[m][k] * W[n][k] with a fused epilogue
+// ---------------------------------------------------------------------------
+enum EpMode {
+  EP_STORE_F32 = 0,  // out_f32[m*ldo + n] = acc
+  EP_RESID = 1,      // out_f32[m*ldo + n] += acc            (residual stream)
+  EP_SWIGLU = 2,     // 128-row groups [64 gate | 64 up] -> out_t[m*ldt + 64g + f] = silu(g) * u
+  EP_SILU = 3,       // out_t[m*ldt + n] = silu(acc)
+  EP_ARGMAX = 4,     // per 128-row tile: (max, argmax) -> part_val/part_idx[m*n_tiles + tile]
+};
+
+struct EpArgs {
+  int mode;
+  float *out_f32;
+  int ldo;
+  void *out_t;
+  int ldt;
+  float *part_val;
+  int *part_idx;
+  int n_tiles;
+};
+
+// ---------------------------------------------------------------------------
+// decoder dimensions as the kernels see them
+// ---------------------------------------------------------------------------
+struct Dims {
+  int d, hq, hkv, hd, inter, vocab, B, R, page_size, num_pages, max_ctx, pages_per_seq;
+  int n_feat;
+  float rms_eps, ln_eps;
+};
+
+__host__ __device__ __forceinline__ size_t pool_layer_elems(const Dims &D) {
+  return (size_t)D.num_pages * 2 * D.hkv * D.page_size * D.hd;
+}
+// element offset of (page, k|v, kv head, in-page slot) inside one layer of a pool
+__host__ __device__ __forceinline__ size_t pool_off(const Dims &D, int page, int kv, int h, int slot) {
+  return ((((size_t)page * 2 + kv) * D.hkv + h) * D.page_size + slot) * D.hd;
+}
+
+// ---------------------------------------------------------------------------
+// launchers (each returns cudaGetLastError())
+// ---------------------------------------------------------------------------
+cudaError_t gemm_simt(int dtype, const void *W, int N, int K, const void *X, int M, int ldx,
+                      const EpArgs &ep, const int *status, cudaStream_t s);
+
+struct AttnArgs {
+  const void *q;          // [rows][hq][hd]
+  const void *pool;       // one layer of a paged K/V pool
+  const int *page_table;  // [batch][pages_per_seq]
+  const void *bk, *bv;    // block K/V [rows][hkv][hd] (non-causal mode) or null
+  const int *pos;         // [rows] compute position of each row
+  const int *seq_len;     // [batch]
+  int causal;             // 1: keys 0..pos (paged); 0: context 0..n-2 (paged) + block rows
+  int n_splits;
+  float *part;            // [rows][hq][n_splits][hd + 2]
+  void *out;              // [rows][hq * hd]
+};
+cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, const int *status,
+                      cudaStream_t s);
+
+}  // namespace dflow

@@ -1,0 +1,25 @@
+// tcgen05 (5th-generation tensor core) weight-streaming GEMM for bf16.
+#pragma once
+#include "dflow_internal.cuh"
+
+namespace dflow {
+
+// Scratch of the tensor-core GEMM inside the handle's workspace.
+struct TcWorkspace {
+  float *part = nullptr;   // split-K partial tiles
+  int *counters = nullptr; // per-tile arrival counters (left at zero after every launch)
+  size_t part_elems = 0;
+  int n_counters = 0;
+  int sm_count = 0;
+};
+
+// Reserve the GEMM scratch at byte offset `off` of `base` (null base: size only).
+void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max);
+// True when the tensor-core kernel covers this problem (bf16, alignment, sizes).
+bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep);
+// Zero the counters once after the workspace is handed over.
+cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s);
+cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M,
+                    int ldx, const EpArgs &ep, int *status, cudaStream_t s);
+
+}  // namespace dflow
