@@ -1,0 +1,403 @@
+#!/usr/bin/env python
+"""Benchmark of the DFlow round on GB300.
+
+One step = one dflow_round (draft -> verify -> accept/commit -> carry) over the
+whole batch of the Qwen3-8B-shaped workload (bf16 random-init weights, 2048
+uniform-random prompt tokens, block 16, seeded uniform{0..16} forced
+acceptance), inputs resident in HBM.  Weights (18.7 GB per round) exceed L2, so
+no flush is needed between steps.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "draft+verify round latency & committed tokens/s, Qwen3-8B shape; % HBM roofline"
+DEFAULT_CONFIG = "qwen3_8b_b1"
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=56)
+    p.add_argument("--warmup", type=int, default=4)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(synth.CONFIGS))
+    p.add_argument("--relay", type=int, default=1, help="0 runs the DFlash baseline (no carry)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--profile-only", action="store_true", help="warmup + a few steps, no timing legs (for ncu)")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), float(pk["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+# --------------------------------------------------------------------------
+# algorithmic bytes of one round
+# --------------------------------------------------------------------------
+
+
+def round_bytes(cfg, mean_ctx: float) -> dict:
+    """DRAM bytes a round must move at minimum: every weight it reads once, the
+    K/V context it attends over, plus the (small) activations.  bf16."""
+    es = 2 if cfg.dtype == "bf16" else 4
+    d, hd, I, V = cfg.d, cfg.head_dim, cfg.inter, cfg.vocab
+    qkv = (cfg.n_q_heads + 2 * cfg.n_kv_heads) * hd * d
+    layer = qkv + d * cfg.n_q_heads * hd + 2 * I * d + d * I
+    kv_tok = 2 * cfg.n_kv_heads * hd * es
+    target_w = (cfg.n_layers * layer + V * d) * es
+    draft_w = (cfg.draft_layers * layer + V * d + cfg.n_feat * d * d + 3 * d * d + 2 * d * d
+               + cfg.draft_layers * 2 * cfg.n_kv_heads * hd * d) * es
+    R = cfg.rows
+    kv = cfg.batch * ((mean_ctx + R) * cfg.n_layers + mean_ctx * cfg.draft_layers) * kv_tok
+    return dict(weights=target_w + draft_w, kv=kv, total=target_w + draft_w + kv)
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: int):
+        self.gpu, self.proc, self.lines = gpu, None, []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            self.proc.wait(timeout=5)
+
+    def summary(self):
+        sm, mx, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = max(mx, float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle on a bounded sample of the workload
+# --------------------------------------------------------------------------
+
+
+class OracleSample:
+    """The oracle's round on a 1-target-layer, 1-draft-layer copy of the workload
+    (full width, batch and context) whose LM head and embedding keep one in
+    `vocab_div` vocabulary rows.  Timers on the oracle's own calls give the
+    per-layer and LM-head costs, from which the full round's time is
+    extrapolated: + (L-1) target layers, + (Ld-1) draft layers and context
+    appends, and the LM heads scaled back to the full vocabulary."""
+
+    def __init__(self, cfg, vocab_div: int = 32):
+        from oracle import Oracle
+        self.cfg = cfg
+        self.vocab_div = vocab_div
+        self.c1 = cfg.replace(n_layers=1, draft_layers=1, feat_layers=(1,), vocab=cfg.vocab // vocab_div)
+        block = np.random.default_rng(0).standard_normal(1 << 22, dtype=np.float32) * np.float32(0.02)
+        W = {}
+        for name, shape in synth.tensor_shapes(self.c1).items():
+            if len(shape) == 1:
+                W[name] = np.zeros(shape, np.float32) if name == "ln_b" else np.ones(shape, np.float32)
+            else:
+                W[name] = np.resize(block, int(np.prod(shape))).reshape(shape)
+        self.o = Oracle(self.c1, W)
+        lens = synth.prompt_lengths(cfg) + 1
+        self.st0 = self.o.state_from_synthetic(synth.synthetic_state(self.c1, ctx_lens=lens,
+                                                                     n_carry=np.full(cfg.batch, cfg.block // 2)))
+        self.acc = {}
+        for name in ("target_forward", "draft_block", "lm_logits", "feature_projection", "draft_inputs", "ctx_append"):
+            self._wrap(name)
+        self.threads = os.cpu_count()
+
+    def _wrap(self, name):
+        f = getattr(self.o, name)
+
+        def w(*a, **k):
+            t = time.perf_counter()
+            r = f(*a, **k)
+            self.acc[name] = self.acc.get(name, 0.0) + time.perf_counter() - t
+            return r
+        setattr(self.o, name, w)
+
+    def step(self, forced):
+        """One sampled round; returns (extrapolated full-round seconds, committed tokens)."""
+        st = self.st0.copy()
+        self.acc = {}
+        t0 = time.perf_counter()
+        ro = self.o.round(st, forced=list(forced))
+        t = time.perf_counter() - t0
+        a = self.acc
+        lm = a.get("lm_logits", 0.0)
+        t_tlayer = a["target_forward"] - a.get("feature_projection", 0.0) - lm / 2
+        t_dlayer = a["draft_block"] - a.get("draft_inputs", 0.0) - lm / 2
+        c = self.cfg
+        full = (t + (c.n_layers - 1) * t_tlayer + (c.draft_layers - 1) * (t_dlayer + a.get("ctx_append", 0.0))
+                + (self.vocab_div - 1) * lm)
+        return full, int((ro.accept + 1).sum())
+
+    def describe(self):
+        c = self.cfg
+        return (f"oracle round (numpy fp64) on a copy of {c.name} with 1 target + 1 draft layer and 1/"
+                f"{self.vocab_div} of the vocabulary (full width {c.d}, batch {c.batch}, context as the workload); "
+                f"time extrapolated to {c.n_layers}+{c.draft_layers} layers and the full LM head with timers on the "
+                f"oracle's own calls")
+
+
+def run_cpu_sample(cfg, steps: int, warmup: int, sched):
+    s = OracleSample(cfg)
+    for w in range(warmup):
+        s.step(sched[w % len(sched)])
+    tot_t = tot_tok = 0.0
+    for k in range(steps):
+        t, tok = s.step(sched[(warmup + k) % len(sched)])
+        tot_t += t
+        tot_tok += tok
+    return tot_tok / tot_t, tot_t / steps, s
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle on a bounded sample of the workload."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cfg = synth.CONFIGS[args.config]
+    sched = synth.forced_schedule(cfg, args.warmup + args.steps)
+    t0 = time.time()
+    value, sec_per_round, s = run_cpu_sample(cfg, args.steps, args.warmup, sched)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec_per_round * 1e3, 1),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "batch": cfg.batch, "prompt": cfg.prompt_len, "block": cfg.block,
+                   "l2": "inputs larger than L2"},
+        "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "cores": s.threads, "kind": "oracle",
+                         "sample": s.describe()},
+        "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "wall_s": round(time.time() - t0, 1),
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        build.build()
+    if world > 1:
+        dist.barrier()
+
+    cfg = synth.CONFIGS[args.config]
+    K, Wm = args.steps, args.warmup
+    n_rounds = Wm + K
+    lens = synth.prompt_lengths(cfg)
+    max_ctx = cfg.replace(new_tokens=n_rounds * cfg.rows).max_ctx()
+    weights = random_weights(cfg, seed=0)
+    eng = Engine(cfg, weights, max_batch=cfg.batch, max_ctx=max_ctx)
+    st = eng.new_state(cfg.batch, page_seed=rank)
+    prompts = synth.prompts(cfg)
+    eng.prefill(st, prompts)
+    assert eng.read_status(st) == 0, "prefill failed"
+    sched = synth.forced_schedule(cfg, n_rounds, seed=synth.SEED_SCHEDULE + rank)
+    forced_dev = torch.as_tensor(sched).cuda()
+    acc = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
+    comm = torch.empty(cfg.batch, cfg.rows, dtype=torch.int32, device="cuda")
+
+    for w in range(Wm):
+        eng.round(st, forced_dev[w], out=(acc, comm))
+    torch.cuda.synchronize()
+    # snapshot of the per-sequence state after warmup: every leg starts from it
+    snap = {k: getattr(st, k).clone() for k in ("tokens", "seq_len", "carry", "n_carry", "boundary")}
+
+    def restore():
+        for k, v in snap.items():
+            getattr(st, k).copy_(v)
+        torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x: float) -> float:
+        if world == 1:
+            return x
+        t = torch.tensor([x], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    if args.profile_only:
+        # rounds inside a profiler range, for `ncu --profile-from-start off`
+        torch.cuda.cudart().cudaProfilerStart()
+        for k in range(min(K, 2)):
+            eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+        torch.cuda.synchronize()
+        torch.cuda.cudart().cudaProfilerStop()
+        print(json.dumps({"profile_only": True, "launches": eng.launch_count()}))
+        return
+
+    committed = float((sched[Wm:Wm + K] + 1).sum())  # a+1 per sequence per round (forced a)
+    ctx0 = float(snap["seq_len"].float().mean())
+    mean_ctx = ctx0 + float((sched[Wm:Wm + K] + 1).mean()) * K / 2
+
+    # ---- device leg: K rounds back to back, CUDA events on the launching stream
+    restore()
+    stream = torch.cuda.current_stream()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    n0 = eng.launch_count()
+    with ClockSampler(local) as clocks:
+        barrier()
+        ev[0].record(stream)
+        for k in range(K):
+            eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+            ev[k + 1].record(stream)
+        torch.cuda.synchronize()
+    launches = eng.launch_count() - n0
+    assert eng.read_status(st) == 0, "device status set during the timed leg"
+    per = [ev[k].elapsed_time(ev[k + 1]) for k in range(K)]
+    total_ms = max_over_ranks(ev[0].elapsed_time(ev[K]))
+    value = committed * world / (total_ms / 1e3)
+
+    # ---- end-to-end leg: host buffers, H2D of the step's inputs and D2H of its result inside the region
+    e2e = None
+    if not args.no_e2e:
+        restore()
+        h_forced = torch.as_tensor(sched).pin_memory()
+        h_acc = torch.empty(K, cfg.batch, dtype=torch.int32).pin_memory()
+        h_comm = torch.empty(K, cfg.batch, cfg.rows, dtype=torch.int32).pin_memory()
+        d_forced = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for k in range(K):
+            d_forced.copy_(h_forced[Wm + k], non_blocking=True)
+            eng.round(st, d_forced, out=(acc, comm))
+            h_acc[k].copy_(acc, non_blocking=True)
+            h_comm[k].copy_(comm, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1))
+        assert np.array_equal(h_acc.numpy(), sched[Wm:Wm + K]), "accept lengths differ from the schedule"
+        e2e = {"value": round(committed * world / (e2e_ms / 1e3), 2), "unit": "tokens/s",
+               "h2d_bytes_per_step": 4 * cfg.batch, "d2h_bytes_per_step": 4 * cfg.batch * (1 + cfg.rows)}
+
+    # ---- profiled leg: per-launch events around the GEMMs (the dominant kernel)
+    restore()
+    eng.profile(True)
+    for k in range(K):
+        eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+    torch.cuda.synchronize()
+    prof = eng.profile_read()
+    eng.profile(False)
+
+    hbm, tflops, peak_src = peaks()
+    g = prof["gemm"]
+    gemm_gbs = g["bytes"] / (g["ms"] / 1e3) / 1e9 if g["ms"] > 0 else 0.0
+    rb = round_bytes(cfg, mean_ctx)
+    ms_step = total_ms / K
+    round_gbs = rb["total"] / (ms_step / 1e3) / 1e9
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": K, "warmup": Wm,
+        "ms_per_step": round(ms_step, 4), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if cfg.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": cfg.name, "batch": cfg.batch, "prompt": int(lens.max()), "block": cfg.block,
+                   "target_layers": cfg.n_layers, "draft_layers": cfg.draft_layers, "d_model": cfg.d,
+                   "acceptance": f"forced {cfg.schedule}", "relay": bool(args.relay),
+                   "l2": "inputs larger than L2 (weights %.1f GB/round)" % (rb["weights"] / 1e9)},
+        "round_latency_ms": {"mean": round(ms_step, 4), "p10": round(float(np.percentile(per, 10)), 4),
+                             "p50": round(float(np.percentile(per, 50)), 4),
+                             "p90": round(float(np.percentile(per, 90)), 4)},
+        "roofline": {"bound": "hbm", "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(gemm_gbs / hbm, 4), "traffic": None, "kernel": "weight-streaming GEMM",
+                     "peak_source": peak_src, "launches": g["launches"], "avg_launch_us": round(1e3 * g["ms"] / max(1, g["launches"]), 2)},
+        "round_roofline": {"bound": "hbm", "alg_bytes": rb["total"], "achieved": round(round_gbs, 1), "peak": hbm,
+                           "frac": round(round_gbs / hbm, 4), "unit": "GB/s", "peak_source": peak_src},
+        "phase_ms": {"gemm": round(g["ms"] / K, 4), "attention": round(prof["attn"]["ms"] / K, 4)},
+        "gpu_launches": int(launches),
+        "e2e": e2e,
+        "clocks": clocks.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cv, cs, s = run_cpu_sample(cfg, steps=1, warmup=0, sched=sched)
+        line["cpu_baseline"] = {"value": round(cv, 4), "unit": "tokens/s", "cores": s.threads, "kind": "oracle",
+                                "sample": s.describe(), "sec_per_round": round(cs, 2)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

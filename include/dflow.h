@@ -195,6 +195,27 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
 dflow_status dflow_read_status(dflow_handle *h, const dflow_state *st, int32_t *host_status,
                                void *stream);
 
+/* ---- measurement (not part of the method) ----------------------------------
+ * With profiling enabled, the library brackets every launch of a kernel class
+ * with CUDA events on the launching stream and accumulates, per class, the
+ * launch count, the summed event durations and the algorithmic DRAM bytes and
+ * flops of those launches (weights + activations read, outputs written; for
+ * attention the K/V bytes are not known on the host and are left at 0). */
+enum { DFLOW_PROF_GEMM = 0, DFLOW_PROF_ATTN = 1, DFLOW_PROF_OTHER = 2, DFLOW_PROF_N = 3 };
+typedef struct dflow_kernel_profile {
+  int64_t launches;
+  double total_ms;
+  double alg_bytes;
+  double alg_flops;
+} dflow_kernel_profile;
+
+/* Turn per-launch event timing on (1) or off (0); either way clears the record. */
+dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable);
+/* Waits for the recorded events, then fills out[DFLOW_PROF_N]. */
+dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out);
+/* Kernels launched by this handle since creation (always counted). */
+dflow_status dflow_launch_count(const dflow_handle *h, uint64_t *count);
+
 #ifdef __cplusplus
 }
 #endif

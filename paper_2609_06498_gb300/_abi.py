@@ -45,6 +45,13 @@ class State(ctypes.Structure):
                 ("active", ctypes.c_void_p), ("status", ctypes.c_void_p)]
 
 
+class KernelProfile(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_int64), ("total_ms", ctypes.c_double), ("alg_bytes", ctypes.c_double),
+                ("alg_flops", ctypes.c_double)]
+
+
+PROF_GEMM, PROF_ATTN, PROF_OTHER, PROF_N = 0, 1, 2, 3
+
 # (name, argtypes) of every exported function of include/dflow.h
 _P = ctypes.c_void_p
 _SIGS = {
@@ -60,6 +67,9 @@ _SIGS = {
     "dflow_carry_hidden": ([_P, ctypes.POINTER(State), _P, _P, _P, _P], ctypes.c_int),
     "dflow_round": ([_P, ctypes.POINTER(State), _P, _P, _P, ctypes.c_int32, _P], ctypes.c_int),
     "dflow_read_status": ([_P, ctypes.POINTER(State), c_i32p, _P], ctypes.c_int),
+    "dflow_profile_enable": ([_P, ctypes.c_int32], ctypes.c_int),
+    "dflow_profile_read": ([_P, ctypes.POINTER(KernelProfile)], ctypes.c_int),
+    "dflow_launch_count": ([_P, ctypes.POINTER(ctypes.c_uint64)], ctypes.c_int),
 }
 EXPORTS = tuple(_SIGS)
 

@@ -378,6 +378,13 @@ struct dflow_handle {
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
   int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen;
   TcWorkspace tcw;
+  // measurement
+  uint64_t n_launch = 0;
+  bool prof = false;
+  struct ProfRec { cudaEvent_t e0, e1; int kind; double bytes, flops; };
+  std::vector<ProfRec> prof_recs;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_next = 0;
 };
 
 namespace {
@@ -386,6 +393,12 @@ namespace {
   do {                                               \
     cudaError_t e_ = (expr);                         \
     if (e_ != cudaSuccess) return DFLOW_ERR_CUDA;    \
+  } while (0)
+
+#define KL(...)          \
+  do {                   \
+    __VA_ARGS__;         \
+    ++k.h->n_launch;     \
   } while (0)
 
 struct Call {
@@ -442,9 +455,52 @@ int pick_splits(const dflow_handle *h, int batch, int rows) {
   return std::max(1, std::min(std::min(want, cap), 64));
 }
 
+cudaEvent_t prof_event(dflow_handle *h) {
+  if (h->ev_next == h->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    h->ev_pool.push_back(e);
+  }
+  return h->ev_pool[h->ev_next++];
+}
+
+// brackets one launch of class `kind` with events when profiling is on
+struct ProfScope {
+  dflow_handle *h;
+  cudaStream_t s;
+  cudaEvent_t e0 = nullptr;
+  int kind;
+  double bytes, flops;
+  ProfScope(dflow_handle *h_, cudaStream_t s_, int kind_, double bytes_, double flops_)
+      : h(h_), s(s_), kind(kind_), bytes(bytes_), flops(flops_) {
+    if (h->prof && (e0 = prof_event(h))) cudaEventRecord(e0, s);
+  }
+  ~ProfScope() {
+    if (!e0) return;
+    cudaEvent_t e1 = prof_event(h);
+    if (!e1) return;
+    cudaEventRecord(e1, s);
+    h->prof_recs.push_back({e0, e1, kind, bytes, flops});
+  }
+};
+
+double ep_out_bytes(const EpArgs &ep, int M, int N, int esz) {
+  switch (ep.mode) {
+    case EP_STORE_F32: return 4.0 * M * N;
+    case EP_RESID: return 8.0 * M * N;
+    case EP_SWIGLU: return (double)esz * M * N / 2;
+    case EP_SILU: return (double)esz * M * N;
+    case EP_ARGMAX: return 8.0 * M * ((N + 127) / 128);
+  }
+  return 0.0;
+}
+
 cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int M, int ldx,
                  const EpArgs &ep) {
   dflow_handle *h = k.h;
+  const double es = h->esz;
+  ProfScope ps(h, k.s, DFLOW_PROF_GEMM, es * N * K + es * M * K + ep_out_bytes(ep, M, N, h->esz), 2.0 * M * N * K);
+  ++h->n_launch;
   if (h->use_tc && tc_supports(N, K, M, ldx, ep)) return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s);
   return gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, k.status, k.s);
 }
@@ -467,7 +523,7 @@ EpArgs ep_t(int mode, void *out, int ldt) {
 template <typename T>
 cudaError_t rmsnorm(const Call &k, const float *x, int ldx, const float *w, void *y, int ldy, int rows) {
   const Dims &D = k.h->D;
-  k_rmsnorm<T><<<rows, 256, 0, k.s>>>(x, ldx, w, static_cast<T *>(y), ldy, D.d, D.rms_eps, k.status);
+  KL(k_rmsnorm<T><<<rows, 256, 0, k.s>>>(x, ldx, w, static_cast<T *>(y), ldy, D.d, D.rms_eps, k.status));
   return cudaGetLastError();
 }
 
@@ -478,11 +534,11 @@ cudaError_t qkv_post(const Call &k, const Dims &D, int rows, const float *src, i
   const int heads = nq + 2 * D.hkv;
   dim3 grid(rows, (heads + 3) / 4);
   if (D.hd == 128)
-    k_qkv_post<T, 128><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
-                                               (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status);
+    KL(k_qkv_post<T, 128><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+                                               (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status));
   else
-    k_qkv_post<T, 64><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
-                                              (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status);
+    KL(k_qkv_post<T, 64><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+                                              (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status));
   return cudaGetLastError();
 }
 
@@ -515,7 +571,11 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
   a.n_splits = splits;
   a.part = h->apart;
   a.out = h->ao;
-  if ((e = attention(h->dtype, D, batch, a, k.status, k.s))) return e;
+  {
+    ProfScope ps(h, k.s, DFLOW_PROF_ATTN, 0.0, 4.0 * rows * D.hq * D.hd);
+    h->n_launch += 2;
+    if ((e = attention(h->dtype, D, batch, a, k.status, k.s))) return e;
+  }
   if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, ep_f32(h->x, D.d, EP_RESID)))) return e;
   if ((e = rmsnorm<T>(k, h->x, D.d, L.mlp_norm, h->xn, D.d, rows))) return e;
   if ((e = gemm(k, L.w_gate_up, 2 * D.inter, D.d, h->xn, rows, D.d, ep_t(EP_SWIGLU, h->mlp, D.inter)))) return e;
@@ -535,7 +595,7 @@ cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *
   ep.part_idx = h->am_idx;
   ep.n_tiles = h->vocab_tiles;
   if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
-  k_argmax_reduce<<<(rows + 7) / 8, 256, 0, k.s>>>(h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status);
+  KL(k_argmax_reduce<<<(rows + 7) / 8, 256, 0, k.s>>>(h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status));
   if ((e = cudaGetLastError())) return e;
   if (logits) return gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep_f32(logits, D.vocab));
   return cudaSuccess;
@@ -554,7 +614,7 @@ cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_
     if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits))) return e;
     for (int fi = 0; fi < D.n_feat; ++fi) {
       if (h->cfg.feat_layers[fi] == l + 1) {
-        k_stash<T><<<rows, 256, 0, k.s>>>(h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status);
+        KL(k_stash<T><<<rows, 256, 0, k.s>>>(h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status));
         if ((e = cudaGetLastError())) return e;
         ++f;
       }
@@ -595,19 +655,19 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R, B = D.B;
-  k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status);
+  KL(k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status));
   CK(cudaGetLastError());
   if (relay) {
     // Eq. 4 for every slot of every sequence; Eq. 5 keeps slots j <= n_carry
-    k_relay_u<T><<<batch * B, 256, 0, k.s>>>((const T *)h->w.embed, st->boundary, (const T *)st->carry,
-                                             (T *)h->relay_u, D.d, B, D.vocab, k.status);
+    KL(k_relay_u<T><<<batch * B, 256, 0, k.s>>>((const T *)h->w.embed, st->boundary, (const T *)st->carry,
+                                             (T *)h->relay_u, D.d, B, D.vocab, k.status));
     CK(cudaGetLastError());
     CK(gemm(k, h->w.relay_w1, D.d, 3 * D.d, h->relay_u, batch * B, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)));
     CK(gemm(k, h->w.relay_w2, 2 * D.d, D.d, h->relay_h, batch * B, D.d, ep_f32(h->gf32, 2 * D.d)));
   }
-  k_draft_input<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
+  KL(k_draft_input<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
                                           h->cfg.max_ctx, (const T *)st->carry, st->n_carry, h->gf32,
-                                          h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B, k.status);
+                                          h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B, k.status));
   CK(cudaGetLastError());
   const int splits = pick_splits(h, batch, rows);
   for (int l = 0; l < h->cfg.draft_layers; ++l) {
@@ -615,8 +675,8 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
     CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits));
   }
   CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
-  k_draft_out<<<(rows + 127) / 128, 128, 0, k.s>>>(h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
-                                                   D.R, blk, k.status);
+  KL(k_draft_out<<<(rows + 127) / 128, 128, 0, k.s>>>(h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
+                                                   D.R, blk, k.status));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
@@ -626,9 +686,9 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status);
+  KL(k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status));
   CK(cudaGetLastError());
-  k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w);
+  KL(k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w));
   CK(cudaGetLastError());
   CK(target_forward<T>(k, D, batch, st, g, feats, logits, pick_splits(h, batch, rows)));
   return DFLOW_OK;
@@ -637,8 +697,8 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
 dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
                        int *acc, int *comm) {
   dflow_handle *h = k.h;
-  k_accept<<<(st->batch + 31) / 32, 32, 0, k.s>>>(blk, g, forced, st->tokens, st->seq_len, st->active,
-                                                 st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w);
+  KL(k_accept<<<(st->batch + 31) / 32, 32, 0, k.s>>>(blk, g, forced, st->tokens, st->seq_len, st->active,
+                                                 st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
@@ -649,21 +709,21 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  k_carry_rows<<<(rows + 127) / 128, 128, 0, k.s>>>(acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status);
+  KL(k_carry_rows<<<(rows + 127) / 128, 128, 0, k.s>>>(acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status));
   CK(cudaGetLastError());
   CK(ctx_append<T>(k, D, rows, st, feats));
-  k_carry<T><<<dim3(batch, D.B), 256, 0, k.s>>>((const T *)feats, acc, blk, st->tokens, st->seq_len,
+  KL(k_carry<T><<<dim3(batch, D.B), 256, 0, k.s>>>((const T *)feats, acc, blk, st->tokens, st->seq_len,
                                                h->cfg.max_ctx, (T *)st->carry, st->n_carry, st->boundary,
-                                               D.d, D.B, relay, k.status);
+                                               D.d, D.B, relay, k.status));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
 
 dflow_status guard(const Call &k, dflow_state *st) {
   dflow_handle *h = k.h;
-  k_guard<<<(st->batch + 127) / 128, 128, 0, k.s>>>(st->tokens, st->seq_len, st->n_carry, st->boundary,
+  KL(k_guard<<<(st->batch + 127) / 128, 128, 0, k.s>>>(st->tokens, st->seq_len, st->n_carry, st->boundary,
                                                    st->active, st->batch, h->R, h->cfg.max_ctx,
-                                                   h->D.vocab, h->D.B, k.status_w);
+                                                   h->D.vocab, h->D.B, k.status_w));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
@@ -679,15 +739,15 @@ dflow_status do_prefill(const Call &k, dflow_state *st, const int *prompt, int s
   CK(cudaMemcpyAsync(h->plen, plen_host, sizeof(int) * batch, cudaMemcpyHostToDevice, k.s));
   const int splits = pick_splits(h, batch, rows);
   for (int c0 = 0; c0 < maxlen; c0 += PF) {
-    k_rows_prefill<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, h->plen, batch, c0, k.status);
+    KL(k_rows_prefill<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, h->plen, batch, c0, k.status));
     CK(cudaGetLastError());
-    k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
-                                      D.vocab, k.status_w);
+    KL(k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
+                                      D.vocab, k.status_w));
     CK(cudaGetLastError());
     CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, splits));
-    k_prefill_commit<<<(rows + 127) / 128, 128, 0, k.s>>>(prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
+    KL(k_prefill_commit<<<(rows + 127) / 128, 128, 0, k.s>>>(prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
                                                           h->cfg.max_ctx, st->tokens, st->seq_len,
-                                                          st->n_carry, st->boundary, k.status);
+                                                          st->n_carry, st->boundary, k.status));
     CK(cudaGetLastError());
     CK(cudaMemcpyAsync(h->pos2, h->pos, sizeof(int) * rows, cudaMemcpyDeviceToDevice, k.s));
     CK(cudaMemcpyAsync(h->wr2, h->wr, sizeof(int) * rows, cudaMemcpyDeviceToDevice, k.s));
@@ -830,6 +890,7 @@ dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes) {
 
 dflow_status dflow_destroy(dflow_handle *h) {
   if (!h) return DFLOW_ERR_INVALID_ARG;
+  for (cudaEvent_t e : h->ev_pool) cudaEventDestroy(e);
   delete h;
   return DFLOW_OK;
 }
@@ -906,6 +967,36 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
   if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
   if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return r;
   return do_carry<float>(k, st, h->blk, h->feats, accept_len, relay);
+}
+
+dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable) {
+  if (!h) return DFLOW_ERR_INVALID_ARG;
+  h->prof = enable != 0;
+  h->prof_recs.clear();
+  h->ev_next = 0;
+  return DFLOW_OK;
+}
+
+dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out) {
+  if (!h || !out) return DFLOW_ERR_INVALID_ARG;
+  for (int i = 0; i < DFLOW_PROF_N; ++i) out[i] = dflow_kernel_profile{0, 0.0, 0.0, 0.0};
+  for (auto &r : h->prof_recs) {
+    CK(cudaEventSynchronize(r.e1));
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, r.e0, r.e1));
+    dflow_kernel_profile &o = out[r.kind];
+    o.launches += 1;
+    o.total_ms += ms;
+    o.alg_bytes += r.bytes;
+    o.alg_flops += r.flops;
+  }
+  return DFLOW_OK;
+}
+
+dflow_status dflow_launch_count(const dflow_handle *h, uint64_t *count) {
+  if (!h || !count) return DFLOW_ERR_INVALID_ARG;
+  *count = h->n_launch;
+  return DFLOW_OK;
 }
 
 dflow_status dflow_read_status(dflow_handle *h, const dflow_state *st, int32_t *host_status, void *stream) {

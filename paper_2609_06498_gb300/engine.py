@@ -255,6 +255,20 @@ class Engine:
              ctypes.c_void_p(comm.data_ptr()), int(relay), self._stream())
         return acc, comm
 
+    def profile(self, enable: bool) -> None:
+        call("dflow_profile_enable", self.h, int(enable))
+
+    def profile_read(self):
+        out = (_abi.KernelProfile * _abi.PROF_N)()
+        call("dflow_profile_read", self.h, out)
+        return {k: dict(launches=out[i].launches, ms=out[i].total_ms, bytes=out[i].alg_bytes, flops=out[i].alg_flops)
+                for i, k in enumerate(("gemm", "attn", "other"))}
+
+    def launch_count(self) -> int:
+        v = ctypes.c_uint64()
+        call("dflow_launch_count", self.h, ctypes.byref(v))
+        return v.value
+
     def read_status(self, st: DeviceState) -> int:
         v = ctypes.c_int32()
         call("dflow_read_status", self.h, ctypes.byref(st.c), ctypes.byref(v), self._stream())
