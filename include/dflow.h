@@ -211,6 +211,18 @@ typedef struct dflow_kernel_profile {
 
 /* Turn per-launch event timing on (1) or off (0); either way clears the record. */
 dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable);
+/* Test hook: one projection out[m][n] = sum_k X[m][k] W[n][k] through the
+ * library's GEMM kernels (path 0: CUDA-core kernel, path 1: tcgen05 kernel,
+ * bf16 handles only), with the epilogue `mode`: 0 store fp32 out[M][ldo];
+ * 1 add into fp32 out[M][ldo]; 2 SwiGLU of 128-row [64 gate | 64 up] groups
+ * into model-dtype out[M][ldo] (N/2 features); 3 SiLU into model-dtype out;
+ * 4 greedy argmax over n into int32 out[M] (M <= max_batch * max(B+1, 64)).
+ * Uses the handle's workspace; asynchronous on `stream`; device errors go to
+ * *status (int32 device word). */
+dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int32_t N, int32_t K,
+                              const void *X, int32_t M, int32_t ldx, int32_t mode, void *out,
+                              int32_t ldo, int32_t *status, void *stream);
+
 /* Waits for the recorded events, then fills out[DFLOW_PROF_N]. */
 dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out);
 /* Kernels launched by this handle since creation (always counted). */

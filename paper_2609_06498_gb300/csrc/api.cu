@@ -445,7 +445,8 @@ size_t layout(dflow_handle *h, char *base) {
   h->comm = (int *)take(rm * 4);
   h->plen = (int *)take((size_t)c.max_batch * 4);
   h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
-  tc_layout(h->tcw, base, off, h->sm_count, rm);
+  const int max_n = std::max(std::max(D.vocab, 2 * D.inter), std::max(h->gld, D.d));
+  tc_layout(h->tcw, base, off, h->sm_count, rm, (max_n + 127) / 128);
   return off;
 }
 
@@ -989,6 +990,40 @@ dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out) {
     o.total_ms += ms;
     o.alg_bytes += r.bytes;
     o.alg_flops += r.flops;
+  }
+  return DFLOW_OK;
+}
+
+dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int32_t N, int32_t K, const void *X,
+                              int32_t M, int32_t ldx, int32_t mode, void *out, int32_t ldo, int32_t *status,
+                              void *stream) {
+  if (!h || !h->ws || !W || !X || !out || !status || N < 1 || K < 1 || M < 1 || ldx < K) return DFLOW_ERR_INVALID_ARG;
+  if (path == 1 && (!h->use_tc || h->dtype != DFLOW_BF16)) return DFLOW_ERR_UNSUPPORTED;
+  if (mode < 0 || mode > 4) return DFLOW_ERR_INVALID_ARG;
+  if (mode == EP_ARGMAX && ((N + 127) / 128 > h->vocab_tiles || M > h->rows_max)) return DFLOW_ERR_INVALID_ARG;
+  if (K % 32) return DFLOW_ERR_UNSUPPORTED;
+  cudaStream_t s = (cudaStream_t)stream;
+  EpArgs ep{};
+  ep.mode = mode;
+  if (mode == EP_STORE_F32 || mode == EP_RESID) {
+    ep.out_f32 = static_cast<float *>(out);
+    ep.ldo = ldo;
+  } else if (mode == EP_SWIGLU || mode == EP_SILU) {
+    ep.out_t = out;
+    ep.ldt = ldo;
+  } else {
+    ep.part_val = h->am_val;
+    ep.part_idx = h->am_idx;
+    ep.n_tiles = (N + 127) / 128;
+  }
+  cudaError_t e = (path == 1) ? (tc_supports(N, K, M, ldx, ep) ? gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, status, s)
+                                                              : cudaErrorNotSupported)
+                              : gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, status, s);
+  if (e == cudaErrorNotSupported) return DFLOW_ERR_UNSUPPORTED;
+  CK(e);
+  if (mode == EP_ARGMAX) {
+    k_argmax_reduce<<<(M + 7) / 8, 256, 0, s>>>(h->am_val, h->am_idx, ep.n_tiles, M, static_cast<int *>(out), status);
+    CK(cudaGetLastError());
   }
   return DFLOW_OK;
 }

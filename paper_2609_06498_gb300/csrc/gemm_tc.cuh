@@ -14,7 +14,7 @@ struct TcWorkspace {
 };
 
 // Reserve the GEMM scratch at byte offset `off` of `base` (null base: size only).
-void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max);
+void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max, int max_tiles);
 // True when the tensor-core kernel covers this problem (bf16, alignment, sizes).
 bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep);
 // Zero the counters once after the workspace is handed over.

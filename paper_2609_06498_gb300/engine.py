@@ -264,6 +264,16 @@ class Engine:
         return {k: dict(launches=out[i].launches, ms=out[i].total_ms, bytes=out[i].alg_bytes, flops=out[i].alg_flops)
                 for i, k in enumerate(("gemm", "attn", "other"))}
 
+    def debug_gemm(self, path: int, W: torch.Tensor, X: torch.Tensor, mode: int, out: torch.Tensor,
+                   status: torch.Tensor, ldx: Optional[int] = None, M: Optional[int] = None):
+        """Test hook: one GEMM with a fused epilogue through the library (see dflow_debug_gemm)."""
+        N, K = W.shape
+        M = X.shape[0] if M is None else M
+        ldx = X.stride(0) if ldx is None else ldx
+        ldo = out.stride(0) if out.dim() > 1 else 1
+        call("dflow_debug_gemm", self.h, int(path), ctypes.c_void_p(W.data_ptr()), N, K, ctypes.c_void_p(X.data_ptr()),
+             M, ldx, int(mode), ctypes.c_void_p(out.data_ptr()), ldo, ctypes.c_void_p(status.data_ptr()), self._stream())
+
     def launch_count(self) -> int:
         v = ctypes.c_uint64()
         call("dflow_launch_count", self.h, ctypes.byref(v))

@@ -1,0 +1,96 @@
+"""The library's two GEMM kernels (tcgen05 tensor-core and CUDA-core) against a
+plain fp32 matmul of the same bf16 inputs, for every fused epilogue, on shapes
+with ragged tails (N not a multiple of 128, M not a multiple of 16, M above
+one 256-row token tile) and with k-blocks split across CTAs."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [  # (N, K, M)
+    (256, 64, 1), (1000, 512, 17), (6144, 4096, 17), (4096, 4096, 32), (24576, 4096, 17), (4096, 12288, 17),
+    (151936, 4096, 17), (2048, 4096, 272), (512, 1472, 48), (384, 3072, 300), (2944, 512, 5),
+]
+
+
+@pytest.fixture(scope="module")
+def eng():
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = synth.ModelConfig(name="gemm_probe", dtype="bf16", d=512, n_layers=1, n_q_heads=4, n_kv_heads=1,
+                            head_dim=128, inter=1472, vocab=151936, draft_layers=1, feat_layers=(1,), block=16,
+                            batch=16, prompt_len=64, new_tokens=16, schedule="uniform")
+    return Engine(cfg, random_weights(cfg), max_batch=16, max_ctx=256)
+
+
+def _inputs(N, K, M, seed):
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    W = (torch.randn(N, K, generator=g, device="cuda") * 0.05).to(torch.bfloat16)
+    X = torch.randn(M, K, generator=g, device="cuda").to(torch.bfloat16)
+    ref = X.float() @ W.float().T  # plain fp32 matmul of the same bf16 values
+    return W, X, ref
+
+
+def _rel(a, b):
+    return float((a - b).abs().max() / b.abs().max())
+
+
+@pytest.mark.parametrize("path", [1, 0], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("N,K,M", SHAPES)
+def test_store_and_resid(eng, path, N, K, M):
+    if path == 0 and N * K > 30_000_000:
+        pytest.skip("CUDA-core kernel only on small shapes")
+    W, X, ref = _inputs(N, K, M, N + K + M)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.full((M, N), float("nan"), device="cuda")
+    eng.debug_gemm(path, W, X, 0, out, st)
+    torch.cuda.synchronize()
+    assert int(st) == 0
+    assert _rel(out, ref) < 1e-5
+    base = torch.randn(M, N, device="cuda")
+    acc = base.clone()
+    eng.debug_gemm(path, W, X, 1, acc, st)
+    torch.cuda.synchronize()
+    assert _rel(acc - base, ref) < 1e-4
+    out2 = torch.empty_like(out)
+    eng.debug_gemm(path, W, X, 0, out2, st)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2), "not deterministic"
+
+
+@pytest.mark.parametrize("path", [1, 0], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("N,K,M", [(2944, 512, 17), (24576, 4096, 17), (3072, 1024, 300)])
+def test_swiglu_and_silu(eng, path, N, K, M):
+    W, X, ref = _inputs(N, K, M, 7 * N + M)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    h = torch.empty(M, N // 2, dtype=torch.bfloat16, device="cuda")
+    eng.debug_gemm(path, W, X, 2, h, st)
+    g = ref.view(M, N // 128, 2, 64)
+    want = (torch.nn.functional.silu(g[:, :, 0]) * g[:, :, 1]).reshape(M, N // 2)
+    s = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    eng.debug_gemm(path, W, X, 3, s, st)
+    torch.cuda.synchronize()
+    assert int(st) == 0
+    assert _rel(h.float(), want) < 1e-2
+    assert _rel(s.float(), torch.nn.functional.silu(ref)) < 1e-2
+
+
+@pytest.mark.parametrize("path", [1, 0], ids=["tcgen05", "simt"])
+@pytest.mark.parametrize("N,K,M", [(1000, 512, 17), (151936, 4096, 17), (151936, 4096, 1)])
+def test_argmax(eng, path, N, K, M):
+    if path == 0 and N > 100000:
+        pytest.skip("CUDA-core kernel only on small shapes")
+    W, X, ref = _inputs(N, K, M, 11 * N + M)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.empty(M, dtype=torch.int32, device="cuda")
+    eng.debug_gemm(path, W, X, 4, out, st)
+    torch.cuda.synchronize()
+    assert int(st) == 0
+    top2 = ref.topk(2, dim=1)
+    safe = (top2.values[:, 0] - top2.values[:, 1]) > 1e-3
+    assert safe.any()
+    assert torch.equal(out.long()[safe], top2.indices[:, 0][safe])
