@@ -575,7 +575,7 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
   {
     ProfScope ps(h, k.s, DFLOW_PROF_ATTN, 0.0, 4.0 * rows * D.hq * D.hd);
     h->n_launch += 2;
-    if ((e = attention(h->dtype, D, batch, a, k.status, k.s))) return e;
+    if ((e = attention(h->dtype, D, batch, a, k.status_w, k.s))) return e;
   }
   if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, ep_f32(h->x, D.d, EP_RESID)))) return e;
   if ((e = rmsnorm<T>(k, h->x, D.d, L.mlp_norm, h->xn, D.d, rows))) return e;

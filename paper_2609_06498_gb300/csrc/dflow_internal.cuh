@@ -105,7 +105,9 @@ struct AttnArgs {
   float *part;            // [rows][hq][n_splits][hd + 2]
   void *out;              // [rows][hq * hd]
 };
-cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, const int *status,
-                      cudaStream_t s);
+cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s);
+// tensor-core path for bf16 caches with 64-token pages (attn_tc.cu)
+bool attention_tc_supported(const Dims &D);
+cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s);
 
 }  // namespace dflow

@@ -1,8 +1,14 @@
 // tcgen05 (5th-generation tensor core) weight-streaming GEMM for bf16.
 #pragma once
+#include <cuda.h>
+
 #include "dflow_internal.cuh"
 
 namespace dflow {
+
+// 2D tensor map of a bf16 row-major [rows][ld] matrix, box 64 columns x box_rows
+// rows, 128-byte swizzle (cached by arguments).
+bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows);
 
 // Scratch of the tensor-core GEMM inside the handle's workspace.
 struct TcWorkspace {
