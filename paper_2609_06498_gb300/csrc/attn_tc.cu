@@ -146,7 +146,10 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
           *reinterpret_cast<uint4 *>(vt + swz(j, c)) = vx;
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&full[stage]);
+        if (lane == 0) {
+          mbar_arrive(&full[stage]);
+          issued[stage] = (int)ph;  // the drain below waits on the latest fill of every stage
+        }
       }
       if (++stage == STAGES) {
         stage = 0;
