@@ -6,27 +6,30 @@
 // out[m][n] = sum_k X[m][k] W[n][k] with few rows m (the B+1 block rows of each
 // sequence) and many output features n.  The kernel computes the transposed
 // product D[n][m] = W[n][:] . X[m][:] so the weight tile is the 128-row A
-// operand and the token rows are the MMA's N dimension (padded to 16):
+// operand and the token rows are the MMA's N dimension (padded to 16).
 //
-//   * W is cut into 128-feature tiles x 64-wide k-blocks ("units").  The units
-//     are split evenly over one CTA per SM (stream-K): a CTA walks a contiguous
-//     run of units, possibly across tile boundaries.
-//   * warp 0 streams W and X k-blocks with TMA (128-byte swizzle) into a ring
-//     of shared-memory stages; warp 1 issues tcgen05.mma (128 x Npad x 16) into
-//     a TMEM accumulator (two buffers, so the epilogue of one tile overlaps the
-//     MMAs of the next); warps 2-5 read the accumulator with tcgen05.ld and run
-//     the fused epilogue.
-//   * A tile finished by one CTA goes straight to the epilogue.  A tile split
-//     across CTAs leaves fp32 partials in the workspace; the last CTA to arrive
-//     on the tile's counter sums them in a fixed order (deterministic) and runs
-//     the epilogue, then resets the counter.  Nobody spins on another CTA.
+//   * The grid is Q clusters of P CTAs (one CTA per SM).  Cluster q owns the
+//     128-feature weight tiles q, q+Q, q+2Q, ...; inside a tile the P CTAs of
+//     the cluster split the K range (split-K) so that P*Q SMs stream weights.
+//   * In each CTA, warp 0 streams W and X k-blocks with TMA (128-byte swizzle)
+//     into a ring of shared-memory stages; warp 1 issues tcgen05.mma
+//     (128 x Npad x 16) into a TMEM accumulator (two buffers, so one tile's
+//     reduction overlaps the next tile's MMAs); warps 2-5 drain the
+//     accumulator with tcgen05.ld.
+//   * Split-K partials meet in distributed shared memory: each CTA parks its
+//     fp32 partial in its own shared memory, signals its peers' mbarriers,
+//     and sums one slice of the token columns over the P partials (in rank
+//     order, so the result is deterministic) before running the fused
+//     epilogue on that slice.  No partial leaves the cluster.
 //   * Every mbarrier wait is bounded (about 2 s of globaltimer); on expiry the
 //     kernel records DFLOW_ERR_DEVICE_TIMEOUT, drains its own copies and MMAs,
 //     frees its TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <map>
 #include <mutex>
+#include <tuple>
 #include <unordered_map>
 
 #include "gemm_tc.cuh"
@@ -39,35 +42,22 @@ namespace {
 using namespace ptx;
 
 constexpr int BM = 128;           // weight rows per tile (MMA M)
-constexpr int BK = 64;            // k elements per unit (128 bytes of bf16: one swizzle row)
+constexpr int BK = 64;            // k elements per k-block (128 bytes of bf16: one swizzle row)
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int MAX_NPAD = 256;
+constexpr int MAX_SPLIT_NPAD = 64;  // split-K (P > 1) only for up to 64 token columns
 constexpr int THREADS = 192;
 constexpr int SMEM_BUDGET = 224 * 1024;
 
-// ---------------------------------------------------------------------------
-// stream-K schedule (identical on host and device)
-// ---------------------------------------------------------------------------
-__host__ __device__ __forceinline__ int cta_start(int c, int U, int C) { return (int)((long long)c * U / C); }
-__host__ __device__ __forceinline__ int cta_of_unit(int u, int U, int C) {
-  int c = (int)(((long long)(u + 1) * C - 1) / U);
-  if (c > C - 1) c = C - 1;
-  while (c + 1 < C && cta_start(c + 1, U, C) <= u) ++c;
-  while (c > 0 && cta_start(c, U, C) > u) --c;
-  return c;
-}
-
 struct Params {
-  int N, K, M, npad, tiles, kb, U, C, stages, tmem_cols, ldx;
+  int N, K, M, npad, T, kb, P, Q, stages, tmem_cols, red_ld;
   uint32_t idesc;
   EpArgs ep;
-  float *part;
-  int *cnt;
   int *status;
 };
 
 struct Smem {
-  uint64_t full[16], empty[16], accf[2], acce[2], drain;
+  uint64_t full[16], empty[16], accf[2], acce[2], ready, freeb, drain;
   uint32_t tmem;
   int flag;
   int abort;
@@ -76,21 +66,34 @@ struct Smem {
   int ri[4][16];
 };
 
-// epilogue on one 16-column chunk; v[j] = D[row r][col c0+j]
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// epilogue on token columns c0 .. c0+nc-1 (nc <= 16) of tile t; v[j] = D[row r][c0+j]
 template <int EP>
 __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t, int r, int sub, int lane, int c0,
-                                               const float *v) {
+                                               int nc, const float *v) {
   const int n = t * BM + r;
   const EpArgs &ep = p.ep;
+  const int cend = min(c0 + nc, p.M);
   if constexpr (EP == EP_STORE_F32 || EP == EP_RESID || EP == EP_SILU) {
     if (n < p.N) {
+      if constexpr (EP == EP_RESID) {
+        float old[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int col = c0 + j;
-        if (col < p.M) {
-          if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
-          if constexpr (EP == EP_RESID) ep.out_f32[(size_t)col * ep.ldo + n] += v[j];
-          if constexpr (EP == EP_SILU) reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_f(v[j]));
+        for (int j = 0; j < 16; ++j)
+          if (c0 + j < cend) old[j] = ep.out_f32[(size_t)(c0 + j) * ep.ldo + n];
+#pragma unroll
+        for (int j = 0; j < 16; ++j)
+          if (c0 + j < cend) ep.out_f32[(size_t)(c0 + j) * ep.ldo + n] = old[j] + v[j];
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int col = c0 + j;
+          if (col < cend) {
+            if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
+            if constexpr (EP == EP_SILU)
+              reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_f(v[j]));
+          }
         }
       }
     }
@@ -105,7 +108,7 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int col = c0 + j;
-        if (col < p.M)
+        if (col < cend)
           reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + t * 64 + r] =
               __float2bfloat16_rn(silu_f(v[j]) * sm.xch[j][r]);
       }
@@ -129,7 +132,7 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
 #pragma unroll
       for (int s = 1; s < 4; ++s) argmax_merge(bv, bi, sm.rv[s][lane], sm.ri[s][lane]);
       const int col = c0 + lane;
-      if (col < p.M) {
+      if (col < cend) {
         ep.part_val[(size_t)col * ep.n_tiles + t] = bv;
         ep.part_idx[(size_t)col * ep.n_tiles + t] = bi;
       }
@@ -145,10 +148,12 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
-  Smem &sm = *reinterpret_cast<Smem *>(ring + (size_t)p.stages * stage_bytes);
+  float *red = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [BM][red_ld] (P > 1)
+  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(red) + (p.P > 1 ? (size_t)BM * p.red_ld * 4 : 0));
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int c = blockIdx.x;
-  const int u0 = cta_start(c, p.U, p.C), u1 = cta_start(c + 1, p.U, p.C);
+  const int rank = p.P > 1 ? (int)cluster_rank() : 0;
+  const int q = blockIdx.x / p.P;
+  const int kr0 = rank * p.kb / p.P, kr1 = (rank + 1) * p.kb / p.P;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.stages; ++s) {
@@ -159,6 +164,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       mbar_init(&sm.accf[b], 1);
       mbar_init(&sm.acce[b], 4);
     }
+    mbar_init(&sm.ready, p.P > 1 ? p.P - 1 : 1);
+    mbar_init(&sm.freeb, p.P > 1 ? p.P - 1 : 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -171,6 +178,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   }
   tc_fence_before();
   __syncthreads();
+  if (p.P > 1) cluster_sync();  // peers' barriers are initialised before anyone signals them
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
 
@@ -182,23 +190,27 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       uint32_t ph = 0;
       int issued_phase[16];
       for (int s = 0; s < 16; ++s) issued_phase[s] = -1;
-      for (int u = u0; u < u1; ++u) {
-        if (!mbar_wait(&sm.empty[stage], ph ^ 1)) {
-          set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
-          atomicExch(&sm.abort, 1);
-          break;
+      bool ok = true;
+      for (int t = q; t < p.T && ok; t += p.Q) {
+        for (int k = kr0; k < kr1; ++k) {
+          if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
+            ok = false;
+            break;
+          }
+          uint8_t *a = ring + (size_t)stage * stage_bytes;
+          mbar_expect_tx(&sm.full[stage], stage_bytes);
+          tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
+          tma_load_2d(a + A_BYTES, &tmX, k * BK, 0, &sm.full[stage], px);
+          issued_phase[stage] = (int)ph;
+          if (++stage == p.stages) {
+            stage = 0;
+            ph ^= 1;
+          }
         }
-        if (*(volatile int *)&sm.abort) break;
-        const int t = u / p.kb, k = u % p.kb;
-        uint8_t *a = ring + (size_t)stage * stage_bytes;
-        mbar_expect_tx(&sm.full[stage], stage_bytes);
-        tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
-        tma_load_2d(a + A_BYTES, &tmX, k * BK, 0, &sm.full[stage], px);
-        issued_phase[stage] = (int)ph;
-        if (++stage == p.stages) {
-          stage = 0;
-          ph ^= 1;
-        }
+      }
+      if (!ok) {
+        set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+        atomicExch(&sm.abort, 1);
       }
       // every copy this thread started has landed before the CTA may exit
       for (int s = 0; s < p.stages; ++s)
@@ -210,23 +222,21 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     if (lane == 0) {
       int stage = 0;
       uint32_t ph = 0;
-      int seg = 0;
       bool ok = true;
-      for (int u = u0; u < u1 && ok;) {
-        const int t = u / p.kb;
-        const int ue = min(u1, (t + 1) * p.kb);
-        const int buf = seg & 1;
-        if (!mbar_wait(&sm.acce[buf], ((seg >> 1) & 1) ^ 1)) { ok = false; break; }
+      int i = 0;
+      for (int t = q; t < p.T && ok; t += p.Q, ++i) {
+        const int buf = i & 1;
+        if (!mbar_wait(&sm.acce[buf], ((i >> 1) & 1) ^ 1)) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem + buf * p.npad;
-        for (int uu = u; uu < ue; ++uu) {
+        for (int k = kr0; k < kr1; ++k) {
           if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
           tc_fence_after();
           const uint32_t a = smem_u32(ring + (size_t)stage * stage_bytes);
           const uint64_t ad = smem_desc(a), bd = smem_desc(a + A_BYTES);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16(d, ad + 2 * kk, bd + 2 * kk, p.idesc, (uu > u || kk > 0) ? 1u : 0u);
+            mma_bf16(d, ad + 2 * kk, bd + 2 * kk, p.idesc, (k > kr0 || kk > 0) ? 1u : 0u);
           mma_commit(&sm.empty[stage]);
           if (++stage == p.stages) {
             stage = 0;
@@ -235,8 +245,6 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         }
         if (!ok) break;
         mma_commit(&sm.accf[buf]);
-        ++seg;
-        u = ue;
       }
       if (!ok) {
         set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
@@ -252,12 +260,18 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
-    int seg = 0;
-    for (int u = u0; u < u1;) {
-      const int t = u / p.kb;
-      const int ue = min(u1, (t + 1) * p.kb);
-      const int buf = seg & 1;
-      if (leader) sm.flag = mbar_wait(&sm.accf[buf], (seg >> 1) & 1) ? 1 : 0;
+    // token columns this CTA finishes after the split-K reduction (multiple of 4)
+    const int w4 = ((p.npad + 4 * p.P - 1) / (4 * p.P)) * 4;
+    const int s0 = min(rank * w4, p.npad), s1 = min(min((rank + 1) * w4, p.npad), p.M);
+    int i = 0;
+    for (int t = q; t < p.T; t += p.Q, ++i) {
+      const int buf = i & 1;
+      if (leader) {
+        int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
+        if (ok && p.P > 1 && i > 0) ok = mbar_wait_cluster(&sm.freeb, (i - 1) & 1) ? 1 : 0;
+        sm.flag = ok;
+      }
+      __syncwarp();
       epi_bar();
       if (!sm.flag) {
         if (leader) {
@@ -268,57 +282,77 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       }
       tc_fence_after();
       const uint32_t acc_addr = lane_addr + buf * p.npad;
-      const bool whole = (u == t * p.kb) && (ue == (t + 1) * p.kb);
       float v[16];
-      if (whole) {
-        for (int c0 = 0; c0 < p.npad; c0 += 16) {
+      if (p.P == 1) {
+        for (int c0 = 0; c0 < p.npad && c0 < p.M; c0 += 16) {
           tmem_ld16(acc_addr + c0, v);
-          epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, v);
+          epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
       } else {
-        // partial tile: park the fp32 partial, count arrivals, the last one finishes the tile
-        const int cf = cta_of_unit(t * p.kb, p.U, p.C), cl = cta_of_unit((t + 1) * p.kb - 1, p.U, p.C);
-        const int slot = 2 * c + (t == u0 / p.kb ? 0 : 1);
-        float *mine = p.part + (size_t)slot * BM * MAX_NPAD;
-        for (int c0 = 0; c0 < p.npad; c0 += 16) {
+        // park this CTA's fp32 partial in its shared memory (row r, contiguous columns)
+        float *mine = red + (size_t)r * p.red_ld;
+        for (int c0 = 0; c0 < p.npad && c0 < p.M; c0 += 16) {
           tmem_ld16(acc_addr + c0, v);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) mine[(size_t)(c0 + j) * BM + r] = v[j];
+          for (int j = 0; j < 16; j += 4)
+            *reinterpret_cast<float4 *>(mine + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
-        __threadfence();
         epi_bar();
-        if (leader) sm.flag = (atomicAdd(&p.cnt[t], 1) == cl - cf) ? 1 : 0;
+        if (leader) {
+          for (int pr = 0; pr < p.P; ++pr)
+            if (pr != rank) mbar_arrive_remote(&sm.ready, (uint32_t)pr);
+          sm.flag = mbar_wait_cluster(&sm.ready, i & 1) ? 1 : 0;
+        }
+        __syncwarp();
         epi_bar();
-        if (sm.flag) {
-          __threadfence();
-          for (int c0 = 0; c0 < p.npad; c0 += 16) {
+        const bool ok = sm.flag != 0;
+        if (ok) {
+          const uint32_t my_row = smem_u32(mine);
+          for (int c0 = s0; c0 < s1; c0 += 16) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
-            for (int cc = cf; cc <= cl; ++cc) {
-              const int s = 2 * cc + (t == cta_start(cc, p.U, p.C) / p.kb ? 0 : 1);
-              const float *src = p.part + (size_t)s * BM * MAX_NPAD;
+            for (int pr = 0; pr < p.P; ++pr) {  // fixed rank order: deterministic sum
+              const uint32_t base = mapa(my_row, (uint32_t)pr);
 #pragma unroll
-              for (int j = 0; j < 16; ++j) v[j] += __ldcg(src + (size_t)(c0 + j) * BM + r);
+              for (int q4 = 0; q4 < 4; ++q4) {
+                if (c0 + 4 * q4 < s1) {
+                  const float4 x = ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4);
+                  v[4 * q4] += x.x;
+                  v[4 * q4 + 1] += x.y;
+                  v[4 * q4 + 2] += x.z;
+                  v[4 * q4 + 3] += x.w;
+                }
+              }
             }
-            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, v);
+            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, min(16, s1 - c0), v);
           }
-          if (leader) p.cnt[t] = 0;
+        }
+        epi_bar();  // this CTA has finished reading every peer's partial
+        if (leader)
+          for (int pr = 0; pr < p.P; ++pr)
+            if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+        if (!ok) {
+          if (leader) {
+            set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+            atomicExch(&sm.abort, 1);
+          }
+          break;
         }
       }
-      epi_bar();  // sm.flag is rewritten by the leader at the top of the next segment
-      ++seg;
-      u = ue;
+      epi_bar();  // sm.flag is rewritten by the leader at the top of the next tile
     }
   }
 
+  __syncwarp();  // lanes that skipped a single-thread role wait for it here
   tc_fence_before();
   __syncthreads();
+  if (p.P > 1) cluster_sync();  // no CTA leaves while a peer may still read its shared memory
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
@@ -329,15 +363,119 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
 // host side
 // ---------------------------------------------------------------------------
 template <int EP>
+cudaError_t ensure_smem_attr() {
+  static bool done = false;
+  if (done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<EP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048);
+  if (e == cudaSuccess) done = true;
+  return e;
+}
+
+template <int EP>
 cudaError_t launch_ep(const CUtensorMap &mw, const CUtensorMap &mx, const Params &p, size_t smem, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<EP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
+  cudaError_t e = ensure_smem_attr<EP>();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.P * p.Q);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  if (p.P > 1) {
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = p.P;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
   }
-  k_gemm_tc<EP><<<p.C, THREADS, smem, s>>>(mw, mx, p);
-  return cudaGetLastError();
+  return cudaLaunchKernelEx(&cfg, k_gemm_tc<EP>, mw, mx, p);
+}
+
+// clusters of P CTAs (with `smem` bytes each) that fit on the device at once
+template <int EP>
+int max_clusters(int P, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::pair<int, size_t>, int> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  auto key = std::make_pair(P, smem);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (ensure_smem_attr<EP>() == cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(P);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = P;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<EP>, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();
+  cache.emplace(key, n);
+  return n;
+}
+
+struct Choice {
+  int P = 0, Q = 0, stages = 0, red_ld = 0;
+  size_t smem = 0;
+};
+
+// split and cluster count minimising the k-blocks each CTA streams (plus a
+// small charge for the in-cluster reduction)
+template <int EP>
+Choice choose(int T, int kb, int npad, int sm_count) {
+  static std::mutex mu;
+  static std::map<std::tuple<int, int, int>, Choice> cache;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(std::make_tuple(T, kb, npad));
+    if (it != cache.end()) return it->second;
+  }
+  const int stage_bytes = A_BYTES + npad * BK * 2;
+  Choice best;
+  long best_cost = -1;
+  for (int P : {1, 2, 3, 4, 6, 8}) {
+    if (P > kb || (P > 1 && npad > MAX_SPLIT_NPAD)) continue;
+    const int red_ld = npad + 4;
+    const size_t red_bytes = P > 1 ? (size_t)BM * red_ld * 4 : 0;
+    int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
+    if (stages > 16) stages = 16;
+    if (stages < 3) continue;
+    const size_t smem = 1024 + (size_t)stages * stage_bytes + red_bytes + sizeof(Smem);
+    int Q = P == 1 ? sm_count : max_clusters<EP>(P, smem);
+    if (Q <= 0) continue;
+    if (Q > T) Q = T;
+    const long rounds = (T + Q - 1) / Q;
+    const long cost = rounds * ((kb + P - 1) / P) + (P > 1 ? 3 : 0);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best.P = P;
+      best.Q = Q;
+      best.stages = stages;
+      best.red_ld = red_ld;
+      best.smem = smem;
+    }
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  cache.emplace(std::make_tuple(T, kb, npad), best);
+  return best;
+}
+
+template <int EP>
+cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_count, cudaStream_t s) {
+  const Choice c = choose<EP>(p.T, p.kb, p.npad, sm_count);
+  if (c.P == 0) return cudaErrorInvalidValue;
+  p.P = c.P;
+  p.Q = c.Q;
+  p.stages = c.stages;
+  p.red_ld = c.red_ld;
+  return launch_ep<EP>(mw, mx, p, c.smem, s);
 }
 
 }  // namespace
@@ -401,15 +539,11 @@ bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, i
 
 
 void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max, int max_tiles) {
+  (void)base;
+  (void)off;
   (void)rows_max;
-  w.sm_count = sm_count;
-  const size_t part_bytes = (size_t)2 * sm_count * BM * MAX_NPAD * 4;
-  w.part = base ? reinterpret_cast<float *>(base + off) : nullptr;
-  w.part_elems = part_bytes / 4;
-  off += (part_bytes + 255) & ~(size_t)255;
-  w.counters = base ? reinterpret_cast<int *>(base + off) : nullptr;
-  w.n_counters = max_tiles;
-  off += ((size_t)max_tiles * 4 + 255) & ~(size_t)255;
+  (void)max_tiles;
+  w.sm_count = sm_count;  // split-K partials stay in distributed shared memory: no global scratch
 }
 
 bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep) {
@@ -418,13 +552,13 @@ bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep) {
 }
 
 cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s) {
-  return cudaMemsetAsync(w.counters, 0, (size_t)w.n_counters * 4, s);
+  (void)w;
+  (void)s;
+  return cudaSuccess;
 }
 
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
                     const EpArgs &ep_in, int *status, cudaStream_t s) {
-  const int tiles = (N + BM - 1) / BM;
-  if (tiles > w.n_counters) return cudaErrorInvalidValue;
   CUtensorMap mw;
   if (!tensor_map(&mw, W, N, K, K, BM)) return cudaErrorInvalidValue;
   for (int m0 = 0; m0 < M; m0 += MAX_NPAD) {
@@ -434,21 +568,12 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
     p.K = K;
     p.M = Mc;
     p.npad = (Mc + 15) / 16 * 16;
-    p.tiles = tiles;
+    p.T = (N + BM - 1) / BM;
     p.kb = K / BK;
-    p.U = tiles * p.kb;
-    p.C = p.U < w.sm_count ? p.U : w.sm_count;
-    const int stage_bytes = A_BYTES + p.npad * BK * 2;
-    p.stages = (SMEM_BUDGET - (int)sizeof(Smem) - 1024) / stage_bytes;
-    if (p.stages > 16) p.stages = 16;
-    if (p.stages < 2) return cudaErrorInvalidValue;
     int cols = 32;
     while (cols < 2 * p.npad) cols <<= 1;
     p.tmem_cols = cols;
-    p.ldx = ldx;
     p.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-    p.part = w.part;
-    p.cnt = w.counters;
     p.status = status;
     EpArgs ep = ep_in;
     if (ep.out_f32) ep.out_f32 += (size_t)m0 * ep.ldo;
@@ -460,14 +585,13 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
     p.ep = ep;
     CUtensorMap mx;
     if (!tensor_map(&mx, static_cast<const bf16 *>(X) + (size_t)m0 * ldx, Mc, K, ldx, p.npad)) return cudaErrorInvalidValue;
-    const size_t smem = 1024 + (size_t)p.stages * stage_bytes + sizeof(Smem);
     cudaError_t e;
     switch (ep.mode) {
-      case EP_STORE_F32: e = launch_ep<EP_STORE_F32>(mw, mx, p, smem, s); break;
-      case EP_RESID: e = launch_ep<EP_RESID>(mw, mx, p, smem, s); break;
-      case EP_SWIGLU: e = launch_ep<EP_SWIGLU>(mw, mx, p, smem, s); break;
-      case EP_SILU: e = launch_ep<EP_SILU>(mw, mx, p, smem, s); break;
-      case EP_ARGMAX: e = launch_ep<EP_ARGMAX>(mw, mx, p, smem, s); break;
+      case EP_STORE_F32: e = run<EP_STORE_F32>(mw, mx, p, w.sm_count, s); break;
+      case EP_RESID: e = run<EP_RESID>(mw, mx, p, w.sm_count, s); break;
+      case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s); break;
+      case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s); break;
+      case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;
