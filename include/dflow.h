@@ -28,8 +28,10 @@
  *     and launch nothing.  Errors found on the device (sequence capacity
  *     exhausted, token id out of range, invalid carried count, a bounded wait
  *     that timed out) are written to *state->status; every later kernel of the
- *     library that sees a nonzero status returns without writing.  Read it
- *     with dflow_read_status.
+ *     library that indexes memory by device state (tokens, positions, pages,
+ *     counts) returns without writing once it sees a nonzero status (the
+ *     dense projections keep running on their fixed workspace buffers).
+ *     Read it with dflow_read_status.
  *   - A handle is not thread safe and serves one stream at a time.
  *   - dtype DFLOW_F32: weights, activations, caches in fp32, fp32 arithmetic.
  *     dtype DFLOW_BF16: weights, caches, features and carry in bf16; fp32

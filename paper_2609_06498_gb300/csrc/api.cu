@@ -50,6 +50,7 @@ __global__ void k_rope_table(float2 *rope, int max_ctx, int hd, double theta) {
 __global__ void k_guard(const int *tokens, const int *seq_len, const int *n_carry,
                         const int *boundary, const int *active, int batch, int R, int max_ctx,
                         int vocab, int B, int *status) {
+  pdl_entry();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch || !active[b]) return;
   const int n = seq_len[b];
@@ -64,8 +65,9 @@ __global__ void k_guard(const int *tokens, const int *seq_len, const int *n_carr
 }
 
 // rows of a round: row b*R+i at position n_b-1+i; writes allowed for active sequences
-__global__ void k_rows_round(int *pos, int *wr, const int *seq_len, const int *active, int batch,
+__global__ void k_rows_round(int *pos, int *wr, int *kvlen, const int *seq_len, const int *active, int batch,
                              int R, const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * R) return;
@@ -73,11 +75,13 @@ __global__ void k_rows_round(int *pos, int *wr, const int *seq_len, const int *a
   const bool ok = active[b] != 0;
   pos[r] = ok ? seq_len[b] - 1 + i : 0;
   wr[r] = ok;
+  if (i == 0) kvlen[b] = ok ? seq_len[b] - 1 + R : 1;  // causal keys 0..n-2+R once the block is written
 }
 
 // rows of prefill step c: row b*PF+i at position c0+i if inside the prompt
-__global__ void k_rows_prefill(int *pos, int *wr, const int *plen, int batch, int c0,
+__global__ void k_rows_prefill(int *pos, int *wr, int *kvlen, const int *plen, int batch, int c0,
                                const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * PF) return;
@@ -85,6 +89,7 @@ __global__ void k_rows_prefill(int *pos, int *wr, const int *plen, int batch, in
   const bool ok = p < plen[b];
   pos[r] = ok ? p : 0;
   wr[r] = ok;
+  if (r % PF == 0) kvlen[b] = plen[b] > c0 ? min(c0 + PF, plen[b]) : 1;
 }
 
 // x[r] = E[tok] (fp32 residual stream); tok = toks[b*stride + i]
@@ -92,6 +97,7 @@ template <typename T>
 __global__ void k_embed(const T *__restrict__ E, const int *__restrict__ toks, int stride, int R,
                         const int *__restrict__ wr, float *__restrict__ x, int d, int vocab,
                         int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x, b = r / R, i = r % R;
   int tok = (wr == nullptr || wr[r]) ? toks[(size_t)b * stride + i] : 0;
@@ -106,6 +112,7 @@ __global__ void k_embed(const T *__restrict__ E, const int *__restrict__ toks, i
 template <typename T>
 __global__ void k_rmsnorm(const float *__restrict__ x, int ldx, const float *__restrict__ w,
                           T *__restrict__ y, int ldy, int d, float eps, const int *status) {
+  pdl_entry();
   if (*status) return;
   __shared__ float red[32];
   const float *xr = x + (size_t)blockIdx.x * ldx;
@@ -128,6 +135,7 @@ k_qkv_post(Dims D, const float *__restrict__ src, int ld, int nq, const float *_
            const int *__restrict__ pos, const int *__restrict__ wr, int R, T *__restrict__ q_out,
            T *__restrict__ pool, const int *__restrict__ page_table, T *__restrict__ bk,
            T *__restrict__ bv, const int *status) {
+  pdl_entry();
   if (*status) return;
   constexpr int J = HD / 32, H2 = HD / 64;
   const int r = blockIdx.x, lane = threadIdx.x % 32;
@@ -178,6 +186,7 @@ k_qkv_post(Dims D, const float *__restrict__ src, int ld, int nq, const float *_
 template <typename T>
 __global__ void k_stash(const float *__restrict__ x, T *__restrict__ stash, int d, int m, int f,
                         const int *status) {
+  pdl_entry();
   if (*status) return;
   const size_t r = blockIdx.x;
   for (int c = threadIdx.x; c < d; c += blockDim.x) stash[r * m * d + (size_t)f * d + c] = from_f<T>(x[r * d + c]);
@@ -186,6 +195,7 @@ __global__ void k_stash(const float *__restrict__ x, T *__restrict__ stash, int 
 // g[r] = argmax over the per-tile partials (ties: lowest token id)
 __global__ void k_argmax_reduce(const float *__restrict__ pv, const int *__restrict__ pi, int n_tiles,
                                 int rows, int *__restrict__ g, const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32, lane = threadIdx.x % 32;
   if (r >= rows) return;
@@ -201,6 +211,7 @@ template <typename T>
 __global__ void k_relay_u(const T *__restrict__ E, const int *__restrict__ boundary,
                           const T *__restrict__ carry, T *__restrict__ u, int d, int B, int vocab,
                           const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x, b = r / B, s = r % B;
   int t0 = boundary[2 * b], t1 = boundary[2 * b + 1];
@@ -224,6 +235,7 @@ __global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__
                               const float *__restrict__ bg, const float *__restrict__ ln_w,
                               const float *__restrict__ ln_b, float ln_eps, int relay,
                               float *__restrict__ x, int d, int B, const int *status) {
+  pdl_entry();
   if (*status) return;
   __shared__ float red[32];
   const int R = B + 1, r = blockIdx.x, b = r / R, j = r % R;
@@ -257,6 +269,7 @@ __global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__
 __global__ void k_draft_out(const int *__restrict__ gd, const int *__restrict__ tokens,
                             const int *__restrict__ seq_len, int max_ctx, int batch, int R,
                             int *__restrict__ blk, const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * R) return;
@@ -269,6 +282,7 @@ __global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
                          const int *__restrict__ forced, int *__restrict__ tokens,
                          int *__restrict__ seq_len, const int *__restrict__ active, int batch, int B,
                          int max_ctx, int *__restrict__ acc, int *__restrict__ comm, int *status) {
+  pdl_entry();
   if (*status) return;
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
@@ -301,6 +315,7 @@ __global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
 // positions of the rows that join the drafter context after a commit
 __global__ void k_carry_rows(const int *__restrict__ acc, const int *__restrict__ seq_len, int batch,
                              int R, int *__restrict__ pos, int *__restrict__ wr, const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * R) return;
@@ -317,6 +332,7 @@ __global__ void k_carry(const T *__restrict__ feats, const int *__restrict__ acc
                         const int *__restrict__ seq_len, int max_ctx, T *__restrict__ carry,
                         int *__restrict__ n_carry, int *__restrict__ boundary, int d, int B,
                         int relay, const int *status) {
+  pdl_entry();
   if (*status) return;
   const int b = blockIdx.x, s = blockIdx.y, R = B + 1, a = acc[b];
   if (a < 0) return;
@@ -339,6 +355,7 @@ __global__ void k_prefill_commit(const int *__restrict__ prompt, int stride,
                                  int max_ctx, int *__restrict__ tokens, int *__restrict__ seq_len,
                                  int *__restrict__ n_carry, int *__restrict__ boundary,
                                  const int *status) {
+  pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * PF || !wr[r]) return;
@@ -376,7 +393,7 @@ struct dflow_handle {
   float *x, *gf32, *apart, *am_val;
   float2 *rope;
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
-  int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen;
+  int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen;
   TcWorkspace tcw;
   // measurement
   uint64_t n_launch = 0;
@@ -444,6 +461,7 @@ size_t layout(dflow_handle *h, char *base) {
   h->acc = (int *)take((size_t)c.max_batch * 4);
   h->comm = (int *)take(rm * 4);
   h->plen = (int *)take((size_t)c.max_batch * 4);
+  h->kvlen = (int *)take((size_t)c.max_batch * 4);
   h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
   const int max_n = std::max(std::max(D.vocab, 2 * D.inter), std::max(h->gld, D.d));
   tc_layout(h->tcw, base, off, h->sm_count, rm, (max_n + 127) / 128);
@@ -524,7 +542,7 @@ EpArgs ep_t(int mode, void *out, int ldt) {
 template <typename T>
 cudaError_t rmsnorm(const Call &k, const float *x, int ldx, const float *w, void *y, int ldy, int rows) {
   const Dims &D = k.h->D;
-  KL(k_rmsnorm<T><<<rows, 256, 0, k.s>>>(x, ldx, w, static_cast<T *>(y), ldy, D.d, D.rms_eps, k.status));
+  KL(klaunch(k_rmsnorm<T>, rows, 256, 0, k.s, x, ldx, w, static_cast<T *>(y), ldy, D.d, D.rms_eps, k.status));
   return cudaGetLastError();
 }
 
@@ -535,10 +553,10 @@ cudaError_t qkv_post(const Call &k, const Dims &D, int rows, const float *src, i
   const int heads = nq + 2 * D.hkv;
   dim3 grid(rows, (heads + 3) / 4);
   if (D.hd == 128)
-    KL(k_qkv_post<T, 128><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+    KL(klaunch(k_qkv_post<T, 128>, grid, 128, 0, k.s, D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
                                                (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status));
   else
-    KL(k_qkv_post<T, 64><<<grid, 128, 0, k.s>>>(D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
+    KL(klaunch(k_qkv_post<T, 64>, grid, 128, 0, k.s, D, src, ld, nq, qn, kn, k.h->rope, pos, wr, D.R,
                                               (T *)q_out, (T *)pool, pt, (T *)bk, (T *)bv, k.status));
   return cudaGetLastError();
 }
@@ -568,6 +586,7 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
   a.bv = causal ? nullptr : h->bv;
   a.pos = h->pos;
   a.seq_len = st->seq_len;
+  a.kvlen = h->kvlen;
   a.causal = causal;
   a.n_splits = splits;
   a.part = h->apart;
@@ -596,7 +615,7 @@ cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *
   ep.part_idx = h->am_idx;
   ep.n_tiles = h->vocab_tiles;
   if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
-  KL(k_argmax_reduce<<<(rows + 7) / 8, 256, 0, k.s>>>(h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status));
+  KL(klaunch(k_argmax_reduce, (rows + 7) / 8, 256, 0, k.s, h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status));
   if ((e = cudaGetLastError())) return e;
   if (logits) return gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep_f32(logits, D.vocab));
   return cudaSuccess;
@@ -615,7 +634,7 @@ cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_
     if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits))) return e;
     for (int fi = 0; fi < D.n_feat; ++fi) {
       if (h->cfg.feat_layers[fi] == l + 1) {
-        KL(k_stash<T><<<rows, 256, 0, k.s>>>(h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status));
+        KL(klaunch(k_stash<T>, rows, 256, 0, k.s, h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status));
         if ((e = cudaGetLastError())) return e;
         ++f;
       }
@@ -656,17 +675,17 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R, B = D.B;
-  KL(k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status));
+  KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch, D.R, k.status));
   CK(cudaGetLastError());
   if (relay) {
     // Eq. 4 for every slot of every sequence; Eq. 5 keeps slots j <= n_carry
-    KL(k_relay_u<T><<<batch * B, 256, 0, k.s>>>((const T *)h->w.embed, st->boundary, (const T *)st->carry,
+    KL(klaunch(k_relay_u<T>, batch * B, 256, 0, k.s, (const T *)h->w.embed, st->boundary, (const T *)st->carry,
                                              (T *)h->relay_u, D.d, B, D.vocab, k.status));
     CK(cudaGetLastError());
     CK(gemm(k, h->w.relay_w1, D.d, 3 * D.d, h->relay_u, batch * B, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)));
     CK(gemm(k, h->w.relay_w2, 2 * D.d, D.d, h->relay_h, batch * B, D.d, ep_f32(h->gf32, 2 * D.d)));
   }
-  KL(k_draft_input<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
+  KL(klaunch(k_draft_input<T>, rows, 256, 0, k.s, (const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
                                           h->cfg.max_ctx, (const T *)st->carry, st->n_carry, h->gf32,
                                           h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B, k.status));
   CK(cudaGetLastError());
@@ -676,7 +695,7 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
     CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits));
   }
   CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
-  KL(k_draft_out<<<(rows + 127) / 128, 128, 0, k.s>>>(h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
+  KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
                                                    D.R, blk, k.status));
   CK(cudaGetLastError());
   return DFLOW_OK;
@@ -687,9 +706,9 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  KL(k_rows_round<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, st->seq_len, st->active, batch, D.R, k.status));
+  KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch, D.R, k.status));
   CK(cudaGetLastError());
-  KL(k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w));
+  KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w));
   CK(cudaGetLastError());
   CK(target_forward<T>(k, D, batch, st, g, feats, logits, pick_splits(h, batch, rows)));
   return DFLOW_OK;
@@ -698,7 +717,7 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
 dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
                        int *acc, int *comm) {
   dflow_handle *h = k.h;
-  KL(k_accept<<<(st->batch + 31) / 32, 32, 0, k.s>>>(blk, g, forced, st->tokens, st->seq_len, st->active,
+  KL(klaunch(k_accept, (st->batch + 31) / 32, 32, 0, k.s, blk, g, forced, st->tokens, st->seq_len, st->active,
                                                  st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w));
   CK(cudaGetLastError());
   return DFLOW_OK;
@@ -710,10 +729,10 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  KL(k_carry_rows<<<(rows + 127) / 128, 128, 0, k.s>>>(acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status));
+  KL(klaunch(k_carry_rows, (rows + 127) / 128, 128, 0, k.s, acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status));
   CK(cudaGetLastError());
   CK(ctx_append<T>(k, D, rows, st, feats));
-  KL(k_carry<T><<<dim3(batch, D.B), 256, 0, k.s>>>((const T *)feats, acc, blk, st->tokens, st->seq_len,
+  KL(klaunch(k_carry<T>, dim3(batch, D.B), 256, 0, k.s, (const T *)feats, acc, blk, st->tokens, st->seq_len,
                                                h->cfg.max_ctx, (T *)st->carry, st->n_carry, st->boundary,
                                                D.d, D.B, relay, k.status));
   CK(cudaGetLastError());
@@ -722,7 +741,7 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
 
 dflow_status guard(const Call &k, dflow_state *st) {
   dflow_handle *h = k.h;
-  KL(k_guard<<<(st->batch + 127) / 128, 128, 0, k.s>>>(st->tokens, st->seq_len, st->n_carry, st->boundary,
+  KL(klaunch(k_guard, (st->batch + 127) / 128, 128, 0, k.s, st->tokens, st->seq_len, st->n_carry, st->boundary,
                                                    st->active, st->batch, h->R, h->cfg.max_ctx,
                                                    h->D.vocab, h->D.B, k.status_w));
   CK(cudaGetLastError());
@@ -740,13 +759,13 @@ dflow_status do_prefill(const Call &k, dflow_state *st, const int *prompt, int s
   CK(cudaMemcpyAsync(h->plen, plen_host, sizeof(int) * batch, cudaMemcpyHostToDevice, k.s));
   const int splits = pick_splits(h, batch, rows);
   for (int c0 = 0; c0 < maxlen; c0 += PF) {
-    KL(k_rows_prefill<<<(rows + 127) / 128, 128, 0, k.s>>>(h->pos, h->wr, h->plen, batch, c0, k.status));
+    KL(klaunch(k_rows_prefill, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, h->plen, batch, c0, k.status));
     CK(cudaGetLastError());
-    KL(k_embed<T><<<rows, 256, 0, k.s>>>((const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
+    KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
                                       D.vocab, k.status_w));
     CK(cudaGetLastError());
     CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, splits));
-    KL(k_prefill_commit<<<(rows + 127) / 128, 128, 0, k.s>>>(prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
+    KL(klaunch(k_prefill_commit, (rows + 127) / 128, 128, 0, k.s, prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
                                                           h->cfg.max_ctx, st->tokens, st->seq_len,
                                                           st->n_carry, st->boundary, k.status));
     CK(cudaGetLastError());
@@ -1022,7 +1041,7 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
   if (e == cudaErrorNotSupported) return DFLOW_ERR_UNSUPPORTED;
   CK(e);
   if (mode == EP_ARGMAX) {
-    k_argmax_reduce<<<(M + 7) / 8, 256, 0, s>>>(h->am_val, h->am_idx, ep.n_tiles, M, static_cast<int *>(out), status);
+    klaunch(k_argmax_reduce, (M + 7) / 8, 256, 0, s, h->am_val, h->am_idx, ep.n_tiles, M, static_cast<int *>(out), status);
     CK(cudaGetLastError());
   }
   return DFLOW_OK;

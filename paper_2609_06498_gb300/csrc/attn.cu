@@ -23,6 +23,7 @@ constexpr int QG = 4 * QPW;  // query rows per pass
 template <typename T, int HD>
 __global__ void __launch_bounds__(128)
 k_attn_split(Dims D, AttnArgs a, const int *__restrict__ status) {
+  pdl_entry();
   if (*status) return;
   constexpr int DPL = HD / 32;  // dims per lane
   __shared__ float Qs[QG][HD];
@@ -146,6 +147,7 @@ k_attn_split(Dims D, AttnArgs a, const int *__restrict__ status) {
 template <typename T, int HD>
 __global__ void k_attn_combine(Dims D, int rows, int n_splits, const float *__restrict__ part,
                                T *__restrict__ out, const int *__restrict__ status) {
+  pdl_entry();
   if (*status) return;
   const int rh = blockIdx.x;  // row * hq + head
   const int c = threadIdx.x;  // dimension
@@ -168,9 +170,9 @@ __global__ void k_attn_combine(Dims D, int rows, int n_splits, const float *__re
 template <typename T, int HD>
 cudaError_t launch(const Dims &D, int batch, const AttnArgs &a, const int *status, cudaStream_t s) {
   dim3 grid(D.hkv, batch, a.n_splits);
-  k_attn_split<T, HD><<<grid, 128, 0, s>>>(D, a, status);
+  klaunch(k_attn_split<T, HD>, grid, 128, 0, s, D, a, status);
   const int rows = batch * D.R;
-  k_attn_combine<T, HD><<<rows * D.hq, HD, 0, s>>>(D, rows, a.n_splits, a.part,
+  klaunch(k_attn_combine<T, HD>, rows * D.hq, HD, 0, s, D, rows, a.n_splits, a.part,
                                                    static_cast<T *>(a.out), status);
   return cudaGetLastError();
 }

@@ -13,7 +13,11 @@
 //     causal mask inside the verify block, keys past the valid context masked
 //     (and their V rows zeroed in registers, so stale pool bytes never reach
 //     the accumulator).
-//   * each split writes (o, m, l); the combine kernel of attn.cu merges them.
+//   * the key splits of one (kv head, sequence, query group) form a thread-
+//     block cluster: each split leaves (o, m, l) in its shared memory and every
+//     CTA merges a slice of the query rows over all splits through
+//     distributed shared memory, writing the final bf16 rows.  One launch per
+//     attention call, no global partials.
 #include <cuda.h>
 
 #include "dflow_internal.cuh"
@@ -29,6 +33,7 @@ using namespace ptx;
 constexpr int QROWS = 80;  // 5 consumer warps x 16 rows
 constexpr int THREADS = 192;
 constexpr int STAGES = 2;
+constexpr int MAX_SPLITS = 8;  // cluster size (portable limit)
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -62,6 +67,8 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {
 template <int HD, bool BLOCK>
 __global__ void __launch_bounds__(THREADS, 2)
 k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroups, int *status) {
+  (void)qgroups;
+  pdl_entry();
   if (*status) return;
   constexpr int TILE = 64 * HD * 2;  // bytes of one K (or V) tile
   constexpr int QS = HD + 8;         // padded Q row (elements)
@@ -72,20 +79,17 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
   bf16 *qs = reinterpret_cast<bf16 *>(ring + STAGES * 2 * TILE);   // [QROWS][QS]
   uint64_t *full = reinterpret_cast<uint64_t *>(qs + QROWS * QS);
   uint64_t *empty = full + STAGES;
+  float *m_sm = reinterpret_cast<float *>(empty + STAGES);  // [QROWS] running max (base 2) of this split
+  float *l_sm = m_sm + QROWS;                               // [QROWS] softmax denominator of this split
+  float *coef = l_sm + QROWS;                               // [QROWS][MAX_SPLITS] merge weights
+  float *o_sm = reinterpret_cast<float *>(ring);            // [QROWS][HD] after the key loop (reuses the ring)
 
   const int kvh = blockIdx.x, b = blockIdx.y;
-  const int split = blockIdx.z / qgroups, qg = blockIdx.z % qgroups;
+  const int split = blockIdx.z % a.n_splits, qg = blockIdx.z / a.n_splits;  // split = rank in the cluster
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = D.hq / D.hkv, R = D.R, QR = R * G, row0 = qg * QROWS;
 
-  int n_keys;
-  if (a.causal) {
-    int mx = 0;
-    for (int i = 0; i < R; ++i) mx = max(mx, a.pos[b * R + i]);
-    n_keys = mx + 1;
-  } else {
-    n_keys = a.seq_len[b] - 1;
-  }
+  const int n_keys = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;
   const int n_tiles = (n_keys + 63) / 64;
   const int t_lo = (int)((long long)split * n_tiles / a.n_splits);
   const int t_hi = (int)((long long)(split + 1) * n_tiles / a.n_splits);
@@ -159,8 +163,9 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
     if (lane == 0)
       for (int s = 0; s < STAGES; ++s)
         if (issued[s] >= 0 && !mbar_wait(&full[s], (uint32_t)issued[s])) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
-    return;
-  }
+    __syncwarp();
+    __syncthreads();  // (A) every copy into the ring has landed
+  } else {
 
   // ---------------- consumers ----------------
   const int cw = warp - 1;              // 0..4
@@ -310,54 +315,72 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
     }
   }
 
-  // ---- partial result of this split: unnormalised o, max (natural log units), sum
+  // ---- this split's (l) summed over the quad; (m, l) per row to shared memory
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     l[h] += __shfl_xor_sync(0xffffffffu, l[h], 1);
     l[h] += __shfl_xor_sync(0xffffffffu, l[h], 2);
   }
+  __syncthreads();  // (A) the ring is free: reuse it for this split's o
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    const int qr = row0 + cw * 16 + g + 8 * h;
-    if (qr >= QR) continue;
-    const int i = qr / G, head = kvh * G + qr % G;
-    float *dst = a.part + (((size_t)(b * R + i) * D.hq + head) * a.n_splits + split) * (HD + 2);
+    const int rr = cw * 16 + g + 8 * h;
 #pragma unroll
     for (int j = 0; j < HD / 8; ++j)
-      *reinterpret_cast<float2 *>(dst + j * 8 + 2 * t4) = make_float2(o[j][2 * h], o[j][2 * h + 1]);
+      *reinterpret_cast<float2 *>(o_sm + rr * HD + j * 8 + 2 * t4) = make_float2(o[j][2 * h], o[j][2 * h + 1]);
     if (t4 == 0) {
-      dst[HD] = m[h] == -INFINITY ? -INFINITY : m[h] * 0.6931471805599453f;
-      dst[HD + 1] = l[h];
+      m_sm[rr] = m[h];
+      l_sm[rr] = l[h];
     }
   }
-}
+  }  // consumers
 
-template <int HD>
-__global__ void k_combine(Dims D, int n_splits, const float *__restrict__ part, bf16 *__restrict__ out,
-                          const int *__restrict__ status) {
-  if (*status) return;
-  const int rh = blockIdx.x, c = threadIdx.x;
-  const float *p = part + (size_t)rh * n_splits * (HD + 2);
-  float M = -INFINITY;
-  for (int s = 0; s < n_splits; ++s) M = fmaxf(M, p[s * (HD + 2) + HD]);
-  float L = 0.f, acc = 0.f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < n_splits; ++s) {
-      const float ms = p[s * (HD + 2) + HD];
-      if (ms == -INFINITY) continue;
-      const float w = __expf(ms - M);
-      L += w * p[s * (HD + 2) + HD + 1];
-      acc += w * p[s * (HD + 2) + c];
+  // ---- merge the splits of this cluster: CTA `split` finishes rows [r_lo, r_hi)
+  __syncthreads();
+  cluster_sync();
+  const int S = a.n_splits;
+  const int rpr = (QROWS + S - 1) / S;
+  const int r_lo = min(QROWS, split * rpr), r_hi = min(QROWS, r_lo + rpr);
+  for (int rr = r_lo + threadIdx.x; rr < r_hi; rr += THREADS) {
+    float ms[MAX_SPLITS], ls[MAX_SPLITS], M = -INFINITY;
+    for (int sp = 0; sp < S; ++sp) {
+      ms[sp] = ld_dsmem_f32(mapa(smem_u32(m_sm + rr), (uint32_t)sp));
+      ls[sp] = ld_dsmem_f32(mapa(smem_u32(l_sm + rr), (uint32_t)sp));
+      M = fmaxf(M, ms[sp]);
     }
+    float L = 0.f;
+    for (int sp = 0; sp < S; ++sp) L += (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M) * ls[sp];
+    for (int sp = 0; sp < S; ++sp)
+      coef[(rr - r_lo) * MAX_SPLITS + sp] = (ms[sp] == -INFINITY || L <= 0.f) ? 0.f : exp2f(ms[sp] - M) / L;
   }
-  out[(size_t)rh * HD + c] = __float2bfloat16_rn(L > 0.f ? acc / L : 0.f);
+  __syncthreads();
+  bf16 *out = static_cast<bf16 *>(a.out);
+  for (int e = threadIdx.x; e < (r_hi - r_lo) * (HD / 4); e += THREADS) {
+    const int rr = r_lo + e / (HD / 4), d4 = (e % (HD / 4)) * 4, qr = row0 + rr;
+    if (qr >= QR) continue;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int sp = 0; sp < S; ++sp) {
+      const float c = coef[(rr - r_lo) * MAX_SPLITS + sp];
+      const float4 x = ld_dsmem_f4(mapa(smem_u32(o_sm + rr * HD + d4), (uint32_t)sp));
+      acc.x += c * x.x;
+      acc.y += c * x.y;
+      acc.z += c * x.z;
+      acc.w += c * x.w;
+    }
+    const int i = qr / G, head = kvh * G + qr % G;
+    bf16 *dst = out + ((size_t)(b * R + i) * D.hq + head) * HD + d4;
+    *reinterpret_cast<__nv_bfloat162 *>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
+    *reinterpret_cast<__nv_bfloat162 *>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
+  }
+  cluster_sync();  // peers may still read this CTA's shared memory until here
 }
 
 template <int HD, bool BLOCK>
 cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
                    cudaStream_t s) {
   constexpr int TILE = 64 * HD * 2;
-  const size_t smem = 1024 + STAGES * 2 * TILE + QROWS * (HD + 8) * 2 + 4 * STAGES * 8;
+  const size_t smem = 1024 + STAGES * 2 * TILE + QROWS * (HD + 8) * 2 + 4 * STAGES * 8 +
+                      (2 * QROWS + QROWS * MAX_SPLITS) * 4;
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_attn_tc<HD, BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -366,10 +389,21 @@ cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnAr
   }
   const int G = D.hq / D.hkv;
   const int qgroups = (D.R * G + QROWS - 1) / QROWS;
-  dim3 grid(D.hkv, batch, a.n_splits * qgroups);
-  k_attn_tc<HD, BLOCK><<<grid, THREADS, smem, s>>>(tm, D, a, qgroups, status);
-  k_combine<HD><<<batch * D.R * D.hq, HD, 0, s>>>(D, a.n_splits, a.part, static_cast<bf16 *>(a.out), status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(D.hkv, batch, a.n_splits * qgroups);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = 1;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = a.n_splits;
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, k_attn_tc<HD, BLOCK>, tm, D, a, qgroups, status);
 }
 
 }  // namespace
@@ -378,7 +412,9 @@ bool attention_tc_supported(const Dims &D) {
   return D.page_size == 64 && (D.hd == 64 || D.hd == 128);
 }
 
-cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s) {
+cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *status, cudaStream_t s) {
+  AttnArgs a = a_in;
+  a.n_splits = D.pages_per_seq < MAX_SPLITS ? (D.pages_per_seq < 1 ? 1 : D.pages_per_seq) : MAX_SPLITS;
   CUtensorMap tm;
   const int rows = D.num_pages * 2 * D.hkv * D.page_size;
   if (!tensor_map(&tm, a.pool, rows, D.hd, D.hd, 64)) return cudaErrorInvalidValue;

@@ -45,8 +45,34 @@ __device__ __forceinline__ void warp_argmax(float &v, int &i) {
   }
 }
 
+// Programmatic dependent launch: the next kernel of the stream may start as
+// soon as every CTA of this one has begun; griddepcontrol.wait blocks until the
+// previous kernel has finished and its writes are visible.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_entry() {
+  pdl_wait();
+  pdl_trigger();
+}
+
 // first device-detected error wins
 __device__ __forceinline__ void set_status(int *status, int code) { atomicCAS(status, 0, code); }
+
+// launch with programmatic stream serialisation (the kernel must begin with pdl_entry)
+template <typename Kern, typename... Args>
+inline cudaError_t klaunch(Kern kernel, dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
 
 // ---------------------------------------------------------------------------
 // GEMM: out[m][n] = sum_k X[m][k] * W[n][k] with a fused epilogue
@@ -100,6 +126,7 @@ struct AttnArgs {
   const void *bk, *bv;    // block K/V [rows][hkv][hd] (non-causal mode) or null
   const int *pos;         // [rows] compute position of each row
   const int *seq_len;     // [batch]
+  const int *kvlen;       // [batch] causal mode: keys 0..kvlen-1 hold data
   int causal;             // 1: keys 0..pos (paged); 0: context 0..n-2 (paged) + block rows
   int n_splits;
   float *part;            // [rows][hq][n_splits][hd + 2]

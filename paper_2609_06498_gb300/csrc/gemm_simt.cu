@@ -16,6 +16,7 @@ template <typename T, int EP>
 __global__ void __launch_bounds__(256)
 k_gemm_simt(const T *__restrict__ W, const T *__restrict__ X, int N, int K, int M, int ldx,
             EpArgs ep, const int *__restrict__ status) {
+  pdl_entry();
   if (*status) return;
   __shared__ float Ws[TN][TK + 1];
   __shared__ float Xs[TM][TK + 1];
@@ -95,11 +96,11 @@ cudaError_t launch(const void *W, int N, int K, const void *X, int M, int ldx, c
   const T *w = static_cast<const T *>(W);
   const T *x = static_cast<const T *>(X);
   switch (ep.mode) {
-    case EP_STORE_F32: k_gemm_simt<T, EP_STORE_F32><<<grid, 256, 0, s>>>(w, x, N, K, M, ldx, ep, status); break;
-    case EP_RESID: k_gemm_simt<T, EP_RESID><<<grid, 256, 0, s>>>(w, x, N, K, M, ldx, ep, status); break;
-    case EP_SWIGLU: k_gemm_simt<T, EP_SWIGLU><<<grid, 256, 0, s>>>(w, x, N, K, M, ldx, ep, status); break;
-    case EP_SILU: k_gemm_simt<T, EP_SILU><<<grid, 256, 0, s>>>(w, x, N, K, M, ldx, ep, status); break;
-    case EP_ARGMAX: k_gemm_simt<T, EP_ARGMAX><<<grid, 256, 0, s>>>(w, x, N, K, M, ldx, ep, status); break;
+    case EP_STORE_F32: klaunch(k_gemm_simt<T, EP_STORE_F32>, grid, 256, 0, s, w, x, N, K, M, ldx, ep, status); break;
+    case EP_RESID: klaunch(k_gemm_simt<T, EP_RESID>, grid, 256, 0, s, w, x, N, K, M, ldx, ep, status); break;
+    case EP_SWIGLU: klaunch(k_gemm_simt<T, EP_SWIGLU>, grid, 256, 0, s, w, x, N, K, M, ldx, ep, status); break;
+    case EP_SILU: klaunch(k_gemm_simt<T, EP_SILU>, grid, 256, 0, s, w, x, N, K, M, ldx, ep, status); break;
+    case EP_ARGMAX: klaunch(k_gemm_simt<T, EP_ARGMAX>, grid, 256, 0, s, w, x, N, K, M, ldx, ep, status); break;
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();

@@ -144,7 +144,9 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
 template <int EP>
 __global__ void __launch_bounds__(THREADS, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const Params p) {
-  if (*p.status) return;
+  // the next kernel may launch once every CTA of this one runs; inputs produced by
+  // the previous kernel are read only after pdl_wait() (weights are prefetched before it)
+  pdl_trigger();
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
@@ -191,21 +193,34 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       int issued_phase[16];
       for (int s = 0; s < 16; ++s) issued_phase[s] = -1;
       bool ok = true;
-      for (int t = q; t < p.T && ok; t += p.Q) {
-        for (int k = kr0; k < kr1; ++k) {
-          if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
-            ok = false;
-            break;
-          }
-          uint8_t *a = ring + (size_t)stage * stage_bytes;
-          mbar_expect_tx(&sm.full[stage], stage_bytes);
-          tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
-          tma_load_2d(a + A_BYTES, &tmX, k * BK, 0, &sm.full[stage], px);
-          issued_phase[stage] = (int)ph;
-          if (++stage == p.stages) {
-            stage = 0;
-            ph ^= 1;
-          }
+      const int nk = kr1 - kr0;
+      const int n_units = ((p.T - q + p.Q - 1) / p.Q) * nk;  // (tile, k-block) pairs of this CTA, in order
+      // weight tiles of the first ring do not depend on the previous kernel: start them now
+      const int pre = n_units < p.stages ? n_units : p.stages;
+      for (int u = 0; u < pre; ++u) {
+        mbar_expect_tx(&sm.full[u], stage_bytes);
+        tma_load_2d(ring + (size_t)u * stage_bytes, &tmW, (kr0 + u % nk) * BK, (q + (u / nk) * p.Q) * BM, &sm.full[u], pw);
+        issued_phase[u] = 0;
+      }
+      pdl_wait();
+      for (int u = 0; u < pre; ++u)
+        tma_load_2d(ring + (size_t)u * stage_bytes + A_BYTES, &tmX, (kr0 + u % nk) * BK, 0, &sm.full[u], px);
+      stage = pre % p.stages;
+      ph = pre == p.stages ? 1 : 0;
+      for (int u = pre; u < n_units; ++u) {
+        const int t = q + (u / nk) * p.Q, k = kr0 + u % nk;
+        if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
+          ok = false;
+          break;
+        }
+        uint8_t *a = ring + (size_t)stage * stage_bytes;
+        mbar_expect_tx(&sm.full[stage], stage_bytes);
+        tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
+        tma_load_2d(a + A_BYTES, &tmX, k * BK, 0, &sm.full[stage], px);
+        issued_phase[stage] = (int)ph;
+        if (++stage == p.stages) {
+          stage = 0;
+          ph ^= 1;
         }
       }
       if (!ok) {
@@ -260,6 +275,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
+    pdl_wait();
     // token columns this CTA finishes after the split-K reduction (multiple of 4)
     const int w4 = ((p.npad + 4 * p.P - 1) / (4 * p.P)) * 4;
     const int s0 = min(rank * w4, p.npad), s1 = min(min((rank + 1) * w4, p.npad), p.M);
@@ -380,14 +396,17 @@ cudaError_t launch_ep(const CUtensorMap &mw, const CUtensorMap &mx, const Params
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
   if (p.P > 1) {
-    at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = p.P;
-    at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = 1;
-    cfg.attrs = at;
-    cfg.numAttrs = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = p.P;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.numAttrs = 2;
   }
   return cudaLaunchKernelEx(&cfg, k_gemm_tc<EP>, mw, mx, p);
 }

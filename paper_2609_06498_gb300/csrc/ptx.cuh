@@ -139,6 +139,11 @@ __device__ __forceinline__ float4 ld_dsmem_f4(uint32_t caddr) {
                : "memory");
   return v;
 }
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t caddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(caddr) : "memory");
+  return v;
+}
 // every thread of every CTA of the cluster (warps converged)
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
