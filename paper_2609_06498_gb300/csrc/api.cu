@@ -92,11 +92,32 @@ __global__ void k_rows_prefill(int *pos, int *wr, int *kvlen, const int *plen, i
   if (r % PF == 0) kvlen[b] = plen[b] > c0 ? min(c0 + PF, plen[b]) : 1;
 }
 
-// x[r] = E[tok] (fp32 residual stream); tok = toks[b*stride + i]
+// residual-stream row finished by a small kernel: bf16(x * gain) for the next
+// projection and the squared-norm partial of every 128-feature block
+template <typename T>
+__device__ __forceinline__ void norm_outputs(const float *xr, int r, int d, T *xn, const float *gain, float *ss,
+                                             int ld_ss) {
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, nw = blockDim.x / 32;
+  for (int fb = warp; fb < d / 128; fb += nw) {
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int c = fb * 128 + lane + 32 * k;
+      const float v = xr[c];
+      xn[(size_t)r * d + c] = from_f<T>(v * gain[c]);
+      acc += v * v;
+    }
+    acc = warp_sum(acc);
+    if (lane == 0) ss[(size_t)fb * ld_ss + r] = acc;
+  }
+}
+
+// x[r] = E[tok] (fp32 residual stream); tok = toks[b*stride + i].  With xn set,
+// also the first layer's normalised input (see norm_outputs).
 template <typename T>
 __global__ void k_embed(const T *__restrict__ E, const int *__restrict__ toks, int stride, int R,
-                        const int *__restrict__ wr, float *__restrict__ x, int d, int vocab,
-                        int *status) {
+                        const int *__restrict__ wr, float *__restrict__ x, int d, int vocab, T *__restrict__ xn,
+                        const float *__restrict__ gain, float *__restrict__ ss, int ld_ss, int *status) {
   pdl_entry();
   if (*status) return;
   const int r = blockIdx.x, b = r / R, i = r % R;
@@ -106,6 +127,10 @@ __global__ void k_embed(const T *__restrict__ E, const int *__restrict__ toks, i
     tok = 0;
   }
   for (int c = threadIdx.x; c < d; c += blockDim.x) x[(size_t)r * d + c] = to_f(E[(size_t)tok * d + c]);
+  if (xn != nullptr) {
+    __syncthreads();
+    norm_outputs<T>(x + (size_t)r * d, r, d, xn, gain, ss, ld_ss);
+  }
 }
 
 // y[r] = x[r] / rms(x[r]) * w   (fp32 in, model dtype out)
@@ -226,29 +251,13 @@ __global__ void k_relay_u(const T *__restrict__ E, const int *__restrict__ bound
   }
 }
 
-// drafter inputs (Eq. 5): row 0 = E(anchor); slot j <= n_carry:
-// E_mask + beta * LN(h_j) + gamma; other slots E_mask
+// Eq. 5 for one carried slot j of sequence b
 template <typename T>
-__global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__ e_mask,
-                              const int *__restrict__ tokens, const int *__restrict__ seq_len,
-                              int max_ctx, const T *__restrict__ carry, const int *__restrict__ n_carry,
-                              const float *__restrict__ bg, const float *__restrict__ ln_w,
-                              const float *__restrict__ ln_b, float ln_eps, int relay,
-                              float *__restrict__ x, int d, int B, const int *status) {
-  pdl_entry();
-  if (*status) return;
-  __shared__ float red[32];
-  const int R = B + 1, r = blockIdx.x, b = r / R, j = r % R;
-  float *xr = x + (size_t)r * d;
-  if (j == 0) {
-    const int tok = tokens[(size_t)b * max_ctx + seq_len[b] - 1];
-    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = to_f(E[(size_t)tok * d + c]);
-    return;
-  }
-  if (!relay || j > n_carry[b]) {
-    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = e_mask[c];
-    return;
-  }
+__device__ void draft_relay_row(const T *__restrict__ E, const float *__restrict__ e_mask, const T *__restrict__ carry,
+                                const float *__restrict__ bg, const float *__restrict__ ln_w,
+                                const float *__restrict__ ln_b, float ln_eps, float *__restrict__ xr, int d, int B,
+                                int b, int j, float *red) {
+  (void)E;
   const T *h = carry + ((size_t)b * B + j - 1) * d;
   float s1 = 0.f;
   for (int c = threadIdx.x; c < d; c += blockDim.x) s1 += to_f(h[c]);
@@ -263,6 +272,36 @@ __global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
     const float ln = (to_f(h[c]) - mu) * inv * ln_w[c] + ln_b[c];
     xr[c] = e_mask[c] + beta[c] * ln + gamma[c];
+  }
+}
+
+// drafter inputs (Eq. 5): row 0 = E(anchor); slot j <= n_carry:
+// E_mask + beta * LN(h_j) + gamma; other slots E_mask
+template <typename T>
+__global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__ e_mask,
+                              const int *__restrict__ tokens, const int *__restrict__ seq_len,
+                              int max_ctx, const T *__restrict__ carry, const int *__restrict__ n_carry,
+                              const float *__restrict__ bg, const float *__restrict__ ln_w,
+                              const float *__restrict__ ln_b, float ln_eps, int relay,
+                              float *__restrict__ x, int d, int B, T *__restrict__ xn,
+                              const float *__restrict__ gain, float *__restrict__ ss, int ld_ss,
+                              const int *status) {
+  pdl_entry();
+  if (*status) return;
+  __shared__ float red[32];
+  const int R = B + 1, r = blockIdx.x, b = r / R, j = r % R;
+  float *xr = x + (size_t)r * d;
+  if (j == 0) {
+    const int tok = tokens[(size_t)b * max_ctx + seq_len[b] - 1];
+    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = to_f(E[(size_t)tok * d + c]);
+  } else if (!relay || j > n_carry[b]) {
+    for (int c = threadIdx.x; c < d; c += blockDim.x) xr[c] = e_mask[c];
+  } else {
+    draft_relay_row(E, e_mask, carry, bg, ln_w, ln_b, ln_eps, xr, d, B, b, j, red);
+  }
+  if (xn != nullptr) {
+    __syncthreads();
+    norm_outputs<T>(xr, r, d, xn, gain, ss, ld_ss);
   }
 }
 
@@ -387,10 +426,11 @@ struct dflow_handle {
   int attn_split_round, attn_split_pf;
   size_t attn_entries;
   bool use_tc;
+  bool fused;  // tensor-core GEMMs with folded norms and the fused Q/K/V epilogue
   size_t ws_need = 0, ws_bytes = 0;
   char *ws = nullptr;
   // workspace views
-  float *x, *gf32, *apart, *am_val;
+  float *x, *gf32, *apart, *am_val, *ss;
   float2 *rope;
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
   int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen;
@@ -437,6 +477,7 @@ size_t layout(dflow_handle *h, char *base) {
   const size_t rm = h->rows_max, es = h->esz;
   const int qd = D.hq * D.hd, kvd = D.hkv * D.hd;
   h->x = (float *)take(rm * D.d * 4);
+  h->ss = (float *)take(rm * (D.d / 128) * 4);
   h->gf32 = (float *)take(rm * h->gld * 4);
   h->xn = take(rm * D.d * es);
   h->q = take(rm * qd * es);
@@ -566,18 +607,86 @@ cudaError_t qkv_post(const Call &k, const Dims &D, int rows, const float *src, i
 //               attention over positions 0..pos.
 //   causal = 0: drafter layer; block K/V kept in bk/bv, attention over the
 //               drafter context pool (0..n-2) and the block rows.
+// the input RMSNorm of a projection, folded into its epilogue (fused path)
+EpArgs in_norm(EpArgs e, const dflow_handle *h) {
+  e.in_ss = h->ss;
+  e.in_ss_n = h->D.d / 128;
+  e.ld_ss = h->rows_max;
+  e.in_inv_d = 1.0f / h->D.d;
+  e.in_eps = h->D.rms_eps;
+  return e;
+}
+
+// residual add that also leaves bf16(x * next_gain), the squared-norm
+// partials of x and (optionally) the Eq. 1 stash copy of x
+EpArgs resid_norm(const dflow_handle *h, const float *next_gain, void *stash) {
+  EpArgs e = ep_f32(h->x, h->D.d, EP_RESID);
+  e.out_ss = h->ss;
+  e.ld_ss = h->rows_max;
+  e.out_xn = h->xn;
+  e.ld_xn = h->D.d;
+  e.out_gain = next_gain;
+  e.out_stash = stash;
+  e.ld_stash = h->D.n_feat * h->D.d;
+  return e;
+}
+
+// fused Q/K/V epilogue targets: q to h->q, k/v to the paged pool (pool set) or
+// to the block buffers (pool null)
+EpArgs qkv_ep(const dflow_handle *h, const Dims &D, int nq, const float *qn, const float *kn, const int *pos,
+              const int *wr, void *pool, const int *page_table, bool block) {
+  EpArgs e{};
+  e.mode = EP_QKV;
+  QkvOut &o = e.qkv;
+  o.nq = nq;
+  o.hkv = D.hkv;
+  o.hq_row = D.hq;
+  o.eps = D.rms_eps;
+  o.qn = qn;
+  o.kn = kn;
+  o.rope = h->rope;
+  o.pos = pos;
+  o.wr = wr;
+  o.R = D.R;
+  o.q_out = h->q;
+  o.pool = pool;
+  o.page_table = page_table;
+  o.pages_per_seq = D.pages_per_seq;
+  o.page_size = D.page_size;
+  o.num_pages = D.num_pages;
+  o.bk = block ? h->bk : nullptr;
+  o.bv = block ? h->bv : nullptr;
+  return e;
+}
+
+// One Qwen3 decoder layer over `rows` rows held in h->x (fp32 residual).
+//   causal = 1: target layer; K/V written to the paged pool (rows with wr),
+//               attention over positions 0..pos.
+//   causal = 0: drafter layer; block K/V kept in bk/bv, attention over the
+//               drafter context pool (0..n-2) and the block rows.
+// Fused path (tensor-core GEMMs, 128-dim heads): h->xn / h->ss already hold
+// bf16(x * attn_norm) and the squared norms of x; the layer leaves
+// bf16(x * next_gain) and the new norms for whatever projection comes next.
 template <typename T>
 cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_layer_weights &L,
-                          void *pool_layer, const dflow_state *st, int causal, int splits) {
+                          void *pool_layer, const dflow_state *st, int causal, int splits, const float *next_gain,
+                          void *stash) {
   dflow_handle *h = k.h;
   const int rows = batch * D.R, qkv_dim = (D.hq + 2 * D.hkv) * D.hd, qd = D.hq * D.hd;
   cudaError_t e;
-  if ((e = rmsnorm<T>(k, h->x, D.d, L.attn_norm, h->xn, D.d, rows))) return e;
-  if ((e = gemm(k, L.w_qkv, qkv_dim, D.d, h->xn, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
-  if ((e = qkv_post<T>(k, D, rows, h->gf32, h->gld, D.hq, L.q_norm, L.k_norm, h->pos, h->wr, h->q,
-                       causal ? pool_layer : nullptr, st->page_table, causal ? nullptr : h->bk,
-                       causal ? nullptr : h->bv)))
-    return e;
+  if (h->fused) {
+    EpArgs eq = in_norm(qkv_ep(h, D, D.hq, L.q_norm, L.k_norm, h->pos, h->wr, causal ? pool_layer : nullptr,
+                               st->page_table, !causal),
+                        h);
+    if ((e = gemm(k, L.w_qkv, qkv_dim, D.d, h->xn, rows, D.d, eq))) return e;
+  } else {
+    if ((e = rmsnorm<T>(k, h->x, D.d, L.attn_norm, h->xn, D.d, rows))) return e;
+    if ((e = gemm(k, L.w_qkv, qkv_dim, D.d, h->xn, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
+    if ((e = qkv_post<T>(k, D, rows, h->gf32, h->gld, D.hq, L.q_norm, L.k_norm, h->pos, h->wr, h->q,
+                         causal ? pool_layer : nullptr, st->page_table, causal ? nullptr : h->bk,
+                         causal ? nullptr : h->bv)))
+      return e;
+  }
   AttnArgs a{};
   a.q = h->q;
   a.pool = pool_layer;
@@ -596,10 +705,22 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
     h->n_launch += 2;
     if ((e = attention(h->dtype, D, batch, a, k.status_w, k.s))) return e;
   }
+  if (h->fused) {
+    if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, resid_norm(h, L.mlp_norm, nullptr)))) return e;
+    if ((e = gemm(k, L.w_gate_up, 2 * D.inter, D.d, h->xn, rows, D.d, in_norm(ep_t(EP_SWIGLU, h->mlp, D.inter), h))))
+      return e;
+    return gemm(k, L.w_down, D.d, D.inter, h->mlp, rows, D.inter, resid_norm(h, next_gain, stash));
+  }
   if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, ep_f32(h->x, D.d, EP_RESID)))) return e;
   if ((e = rmsnorm<T>(k, h->x, D.d, L.mlp_norm, h->xn, D.d, rows))) return e;
   if ((e = gemm(k, L.w_gate_up, 2 * D.inter, D.d, h->xn, rows, D.d, ep_t(EP_SWIGLU, h->mlp, D.inter)))) return e;
-  return gemm(k, L.w_down, D.d, D.inter, h->mlp, rows, D.inter, ep_f32(h->x, D.d, EP_RESID));
+  if ((e = gemm(k, L.w_down, D.d, D.inter, h->mlp, rows, D.inter, ep_f32(h->x, D.d, EP_RESID)))) return e;
+  if (stash) {
+    KL(klaunch(k_stash<T>, rows, 256, 0, k.s, h->x, (T *)h->stash, D.d, D.n_feat,
+               (int)(((T *)stash - (T *)h->stash) / D.d), k.status));
+    return cudaGetLastError();
+  }
+  return cudaSuccess;
 }
 
 // final RMSNorm -> LM head -> greedy token per row (and fp32 logits when asked)
@@ -608,17 +729,30 @@ cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *
                            float *logits) {
   dflow_handle *h = k.h;
   cudaError_t e;
-  if ((e = rmsnorm<T>(k, h->x, D.d, norm, h->xn, D.d, rows))) return e;
+  if (!h->fused && (e = rmsnorm<T>(k, h->x, D.d, norm, h->xn, D.d, rows))) return e;
   EpArgs ep{};
   ep.mode = EP_ARGMAX;
   ep.part_val = h->am_val;
   ep.part_idx = h->am_idx;
   ep.n_tiles = h->vocab_tiles;
+  if (h->fused) ep = in_norm(ep, h);
   if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
   KL(klaunch(k_argmax_reduce, (rows + 7) / 8, 256, 0, k.s, h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status));
   if ((e = cudaGetLastError())) return e;
-  if (logits) return gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep_f32(logits, D.vocab));
+  if (logits) {
+    EpArgs el = ep_f32(logits, D.vocab);
+    if (h->fused) el = in_norm(el, h);
+    return gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, el);
+  }
   return cudaSuccess;
+}
+
+// feature slot of target layer l+1 in the Eq. 1 stash, or null
+template <typename T>
+void *stash_slot(const dflow_handle *h, int l) {
+  for (int fi = 0; fi < h->D.n_feat; ++fi)
+    if (h->cfg.feat_layers[fi] == l + 1) return static_cast<T *>(h->stash) + (size_t)fi * h->D.d;
+  return nullptr;
 }
 
 // target forward over h->x (embeddings) at h->pos; writes K/V, g, Eq. 1 features
@@ -627,18 +761,12 @@ cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_
                            void *feats, float *logits, int splits) {
   dflow_handle *h = k.h;
   const int rows = batch * D.R;
+  const int L = h->cfg.n_layers;
   cudaError_t e;
-  int f = 0;
-  for (int l = 0; l < h->cfg.n_layers; ++l) {
+  for (int l = 0; l < L; ++l) {
     T *pool_l = static_cast<T *>(st->kv) + (size_t)l * pool_layer_elems(D);
-    if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits))) return e;
-    for (int fi = 0; fi < D.n_feat; ++fi) {
-      if (h->cfg.feat_layers[fi] == l + 1) {
-        KL(klaunch(k_stash<T>, rows, 256, 0, k.s, h->x, (T *)h->stash, D.d, D.n_feat, fi, k.status));
-        if ((e = cudaGetLastError())) return e;
-        ++f;
-      }
-    }
+    const float *next_gain = l + 1 < L ? h->tl[l + 1].attn_norm : h->w.final_norm;
+    if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits, next_gain, stash_slot<T>(h, l)))) return e;
   }
   if ((e = lm_head_argmax<T>(k, D, rows, h->w.final_norm, g, logits))) return e;
   // Eq. 1: H_T = RMSNorm(W_c [H^l1; ...; H^lm])
@@ -655,8 +783,14 @@ cudaError_t ctx_append(const Call &k, const Dims &D, int rows, const dflow_state
   for (int l = 0; l < h->cfg.draft_layers; ++l) {
     const dflow_layer_weights &L = h->dl[l];
     const T *wkv = static_cast<const T *>(L.w_qkv) + qoff;
-    if ((e = gemm(k, wkv, 2 * D.hkv * D.hd, D.d, feats, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
     T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
+    if (h->fused) {
+      if ((e = gemm(k, wkv, 2 * D.hkv * D.hd, D.d, feats, rows, D.d,
+                    qkv_ep(h, D, 0, nullptr, L.k_norm, h->pos2, h->wr2, pool_l, st->page_table, false))))
+        return e;
+      continue;
+    }
+    if ((e = gemm(k, wkv, 2 * D.hkv * D.hd, D.d, feats, rows, D.d, ep_f32(h->gf32, h->gld)))) return e;
     if ((e = qkv_post<T>(k, D, rows, h->gf32, h->gld, 0, nullptr, L.k_norm, h->pos2, h->wr2, nullptr,
                          pool_l, st->page_table, nullptr, nullptr)))
       return e;
@@ -687,12 +821,16 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
   }
   KL(klaunch(k_draft_input<T>, rows, 256, 0, k.s, (const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
                                           h->cfg.max_ctx, (const T *)st->carry, st->n_carry, h->gf32,
-                                          h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B, k.status));
+                                          h->w.ln_w, h->w.ln_b, D.ln_eps, relay, h->x, D.d, B,
+                                          h->fused ? (T *)h->xn : nullptr, h->dl[0].attn_norm, h->ss, h->rows_max,
+                                          k.status));
   CK(cudaGetLastError());
   const int splits = pick_splits(h, batch, rows);
-  for (int l = 0; l < h->cfg.draft_layers; ++l) {
+  const int Ld = h->cfg.draft_layers;
+  for (int l = 0; l < Ld; ++l) {
     T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
-    CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits));
+    const float *next_gain = l + 1 < Ld ? h->dl[l + 1].attn_norm : h->w.draft_final_norm;
+    CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits, next_gain, nullptr));
   }
   CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
   KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
@@ -708,7 +846,8 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   const int batch = st->batch, rows = batch * D.R;
   KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch, D.R, k.status));
   CK(cudaGetLastError());
-  KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, blk, D.R, D.R, nullptr, h->x, D.d, D.vocab, k.status_w));
+  KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, blk, D.R, D.R, (const int *)nullptr, h->x, D.d,
+             D.vocab, h->fused ? (T *)h->xn : nullptr, h->tl[0].attn_norm, h->ss, h->rows_max, k.status_w));
   CK(cudaGetLastError());
   CK(target_forward<T>(k, D, batch, st, g, feats, logits, pick_splits(h, batch, rows)));
   return DFLOW_OK;
@@ -761,8 +900,9 @@ dflow_status do_prefill(const Call &k, dflow_state *st, const int *prompt, int s
   for (int c0 = 0; c0 < maxlen; c0 += PF) {
     KL(klaunch(k_rows_prefill, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, h->plen, batch, c0, k.status));
     CK(cudaGetLastError());
-    KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, prompt + c0, stride, PF, h->wr, h->x, D.d,
-                                      D.vocab, k.status_w));
+    KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, prompt + c0, stride, PF, (const int *)h->wr,
+               h->x, D.d, D.vocab, h->fused ? (T *)h->xn : nullptr, h->tl[0].attn_norm, h->ss, h->rows_max,
+               k.status_w));
     CK(cudaGetLastError());
     CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, splits));
     KL(klaunch(k_prefill_commit, (rows + 127) / 128, 128, 0, k.s, prompt, stride, h->plen, h->pos, h->wr, h->g, batch,
@@ -883,6 +1023,7 @@ dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow
       h->use_tc = (major == 10 && minor == 3) && getenv("DFLOW_DISABLE_TC") == nullptr;
     cudaGetLastError();
   }
+  h->fused = h->use_tc && c.head_dim == 128;
   h->ws_need = layout(h, nullptr);
   *out = h;
   return DFLOW_OK;

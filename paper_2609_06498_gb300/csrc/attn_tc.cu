@@ -33,7 +33,7 @@ using namespace ptx;
 constexpr int QROWS = 80;  // 5 consumer warps x 16 rows
 constexpr int THREADS = 192;
 constexpr int STAGES = 2;
-constexpr int MAX_SPLITS = 8;  // cluster size (portable limit)
+constexpr int MAX_SPLITS = 16;  // cluster size (non-portable; 2 CTAs fit per SM)
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -171,14 +171,24 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
   const int cw = warp - 1;              // 0..4
   const int g = lane / 4, t4 = lane % 4;
   const bf16 *q = static_cast<const bf16 *>(a.q);
-  for (int e = threadIdx.x - 32; e < QROWS * (HD / 8); e += 160) {
-    const int r = e / (HD / 8), c = e % (HD / 8), qr = row0 + r;
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (qr < QR) {
-      const int i = qr / G, h = kvh * G + qr % G;
-      v = *reinterpret_cast<const uint4 *>(q + ((size_t)(b * R + i) * D.hq + h) * HD + c * 8);
+  {
+    // all of this thread's query chunks are loaded before any is stored
+    constexpr int PER = QROWS * (HD / 8) / 160;
+    uint4 v[PER];
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int e = threadIdx.x - 32 + k * 160, r = e / (HD / 8), c = e % (HD / 8), qr = row0 + r;
+      v[k] = make_uint4(0, 0, 0, 0);
+      if (qr < QR) {
+        const int i = qr / G, h = kvh * G + qr % G;
+        v[k] = __ldg(reinterpret_cast<const uint4 *>(q + ((size_t)(b * R + i) * D.hq + h) * HD + c * 8));
+      }
     }
-    *reinterpret_cast<uint4 *>(qs + r * QS + c * 8) = v;
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+      const int e = threadIdx.x - 32 + k * 160, r = e / (HD / 8), c = e % (HD / 8);
+      *reinterpret_cast<uint4 *>(qs + r * QS + c * 8) = v[k];
+    }
   }
   cons_bar();
   uint32_t qf[HD / 16][4];
@@ -338,34 +348,44 @@ k_attn_tc(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int qgroup
   // ---- merge the splits of this cluster: CTA `split` finishes rows [r_lo, r_hi)
   __syncthreads();
   cluster_sync();
-  const int S = a.n_splits;
-  const int rpr = (QROWS + S - 1) / S;
-  const int r_lo = min(QROWS, split * rpr), r_hi = min(QROWS, r_lo + rpr);
-  for (int rr = r_lo + threadIdx.x; rr < r_hi; rr += THREADS) {
-    float ms[MAX_SPLITS], ls[MAX_SPLITS], M = -INFINITY;
+  // (the cluster always has MAX_SPLITS CTAs, so every loop below unrolls and all
+  // remote loads of a thread are in flight together)
+  constexpr int S = MAX_SPLITS;
+  constexpr int RPR = (QROWS + S - 1) / S;
+  const int r_lo = min(QROWS, split * RPR), r_hi = min(QROWS, r_lo + RPR);
+  if (threadIdx.x < r_hi - r_lo) {
+    const int rr = r_lo + threadIdx.x;
+    float ms[S], ls[S], M = -INFINITY;
+#pragma unroll
     for (int sp = 0; sp < S; ++sp) {
       ms[sp] = ld_dsmem_f32(mapa(smem_u32(m_sm + rr), (uint32_t)sp));
       ls[sp] = ld_dsmem_f32(mapa(smem_u32(l_sm + rr), (uint32_t)sp));
-      M = fmaxf(M, ms[sp]);
     }
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) M = fmaxf(M, ms[sp]);
     float L = 0.f;
+#pragma unroll
     for (int sp = 0; sp < S; ++sp) L += (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M) * ls[sp];
+#pragma unroll
     for (int sp = 0; sp < S; ++sp)
-      coef[(rr - r_lo) * MAX_SPLITS + sp] = (ms[sp] == -INFINITY || L <= 0.f) ? 0.f : exp2f(ms[sp] - M) / L;
+      coef[threadIdx.x * MAX_SPLITS + sp] = (ms[sp] == -INFINITY || L <= 0.f) ? 0.f : exp2f(ms[sp] - M) / L;
   }
   __syncthreads();
   bf16 *out = static_cast<bf16 *>(a.out);
   for (int e = threadIdx.x; e < (r_hi - r_lo) * (HD / 4); e += THREADS) {
     const int rr = r_lo + e / (HD / 4), d4 = (e % (HD / 4)) * 4, qr = row0 + rr;
     if (qr >= QR) continue;
+    float4 x[S];
+#pragma unroll
+    for (int sp = 0; sp < S; ++sp) x[sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + rr * HD + d4), (uint32_t)sp));
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
     for (int sp = 0; sp < S; ++sp) {
       const float c = coef[(rr - r_lo) * MAX_SPLITS + sp];
-      const float4 x = ld_dsmem_f4(mapa(smem_u32(o_sm + rr * HD + d4), (uint32_t)sp));
-      acc.x += c * x.x;
-      acc.y += c * x.y;
-      acc.z += c * x.z;
-      acc.w += c * x.w;
+      acc.x += c * x[sp].x;
+      acc.y += c * x[sp].y;
+      acc.z += c * x[sp].z;
+      acc.w += c * x[sp].w;
     }
     const int i = qr / G, head = kvh * G + qr % G;
     bf16 *dst = out + ((size_t)(b * R + i) * D.hq + head) * HD + d4;
@@ -384,6 +404,7 @@ cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnAr
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_attn_tc<HD, BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_attn_tc<HD, BLOCK>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     attr = true;
   }
@@ -414,7 +435,7 @@ bool attention_tc_supported(const Dims &D) {
 
 cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *status, cudaStream_t s) {
   AttnArgs a = a_in;
-  a.n_splits = D.pages_per_seq < MAX_SPLITS ? (D.pages_per_seq < 1 ? 1 : D.pages_per_seq) : MAX_SPLITS;
+  a.n_splits = MAX_SPLITS;  // one cluster of MAX_SPLITS key splits per (kv head, sequence, query group)
   CUtensorMap tm;
   const int rows = D.num_pages * 2 * D.hkv * D.page_size;
   if (!tensor_map(&tm, a.pool, rows, D.hd, D.hd, 64)) return cudaErrorInvalidValue;

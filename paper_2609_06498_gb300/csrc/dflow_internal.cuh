@@ -83,6 +83,24 @@ enum EpMode {
   EP_SWIGLU = 2,     // 128-row groups [64 gate | 64 up] -> out_t[m*ldt + 64g + f] = silu(g) * u
   EP_SILU = 3,       // out_t[m*ldt + n] = silu(acc)
   EP_ARGMAX = 4,     // per 128-row tile: (max, argmax) -> part_val/part_idx[m*n_tiles + tile]
+  EP_QKV = 5,        // per 128-row tile = one head: q/k RMSNorm + rotary, q to q_out, k/v to the cache
+};
+
+// Targets of the fused Q/K/V epilogue (tensor-core path, head_dim 128).  The
+// output rows are nq query heads, then hkv key heads, then hkv value heads.
+struct QkvOut {
+  int nq, hkv, hq_row;       // q heads in this output; kv heads; q heads per q_out row
+  float eps;                 // q/k RMSNorm epsilon
+  const float *qn, *kn;      // q/k norm gains [128]
+  const float2 *rope;        // [max_ctx][64] (cos, sin)
+  const int *pos, *wr;       // per global row: position, cache write allowed
+  int row0;                  // global row of output column 0
+  int R;                     // rows per sequence
+  void *q_out;               // [rows][hq_row][128]
+  void *pool;                // one layer of a paged pool (when bk == null)
+  const int *page_table;
+  int pages_per_seq, page_size, num_pages;
+  void *bk, *bv;             // block K/V [rows][hkv][128] (drafter) or null
 };
 
 struct EpArgs {
@@ -94,6 +112,20 @@ struct EpArgs {
   float *part_val;
   int *part_idx;
   int n_tiles;
+  // input RMSNorm folded into the epilogue: column m is scaled by
+  // rsqrt(sum_i in_ss[i*ld_ss + m] * inv_d + eps) (the gain is already in X)
+  const float *in_ss;
+  int in_ss_n, ld_ss;
+  float in_inv_d, in_eps;
+  // EP_RESID extras for the updated rows x: squared-norm partial of this
+  // tile's 128 features (out_ss[tile*ld_ss + m]), bf16(x * out_gain) and bf16(x)
+  float *out_ss;
+  void *out_xn;
+  int ld_xn;
+  const float *out_gain;
+  void *out_stash;
+  int ld_stash;
+  QkvOut qkv;
 };
 
 // ---------------------------------------------------------------------------

@@ -64,39 +64,125 @@ struct Smem {
   float xch[16][64];
   float rv[4][16];
   int ri[4][16];
+  float ssred[4][16];
+  float col_scale[MAX_NPAD];
 };
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+// per-column sum over the tile's 128 rows (all epilogue threads call it)
+__device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const float *x, float *out) {
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float t = warp_sum(x[j]);
+    if (lane == 0) sm.ssred[sub][j] = t;
+  }
+  epi_bar();
+#pragma unroll
+  for (int j = 0; j < 16; ++j) out[j] = sm.ssred[0][j] + sm.ssred[1][j] + sm.ssred[2][j] + sm.ssred[3][j];
+  epi_bar();
+}
+
 // epilogue on token columns c0 .. c0+nc-1 (nc <= 16) of tile t; v[j] = D[row r][c0+j]
 template <int EP>
 __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t, int r, int sub, int lane, int c0,
-                                               int nc, const float *v) {
+                                               int nc, float *v) {
   const int n = t * BM + r;
   const EpArgs &ep = p.ep;
   const int cend = min(c0 + nc, p.M);
-  if constexpr (EP == EP_STORE_F32 || EP == EP_RESID || EP == EP_SILU) {
+  if (ep.in_ss) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] *= sm.col_scale[min(c0 + j, MAX_NPAD - 1)];
+  }
+  if constexpr (EP == EP_STORE_F32 || EP == EP_SILU) {
     if (n < p.N) {
-      if constexpr (EP == EP_RESID) {
-        float old[16];
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c0 + j < cend) old[j] = ep.out_f32[(size_t)(c0 + j) * ep.ldo + n];
-#pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c0 + j < cend) ep.out_f32[(size_t)(c0 + j) * ep.ldo + n] = old[j] + v[j];
-      } else {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int col = c0 + j;
-          if (col < cend) {
-            if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
-            if constexpr (EP == EP_SILU)
-              reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_f(v[j]));
-          }
+      for (int j = 0; j < 16; ++j) {
+        const int col = c0 + j;
+        if (col < cend) {
+          if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
+          if constexpr (EP == EP_SILU)
+            reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_f(v[j]));
         }
       }
     }
+  } else if constexpr (EP == EP_RESID) {
+    float x[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      x[j] = (n < p.N && c0 + j < cend) ? ep.out_f32[(size_t)(c0 + j) * ep.ldo + n] : 0.f;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int col = c0 + j;
+      if (n < p.N && col < cend) {
+        x[j] += v[j];
+        ep.out_f32[(size_t)col * ep.ldo + n] = x[j];
+        if (ep.out_xn)
+          reinterpret_cast<bf16 *>(ep.out_xn)[(size_t)col * ep.ld_xn + n] = __float2bfloat16_rn(x[j] * ep.out_gain[n]);
+        if (ep.out_stash)
+          reinterpret_cast<bf16 *>(ep.out_stash)[(size_t)col * ep.ld_stash + n] = __float2bfloat16_rn(x[j]);
+      }
+    }
+    if (ep.out_ss) {
+      float sq[16], tot[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) sq[j] = x[j] * x[j];
+      column_sums(sm, sub, lane, sq, tot);
+      if (r < 16 && c0 + r < cend) ep.out_ss[(size_t)t * ep.ld_ss + c0 + r] = tot[r];
+    }
+  } else if constexpr (EP == EP_QKV) {
+    const QkvOut &o = ep.qkv;
+    const int head = t;
+    const int kind = head < o.nq ? 0 : (head < o.nq + o.hkv ? 1 : 2);  // q, k, v
+    const int kvh = kind == 1 ? head - o.nq : head - o.nq - o.hkv;
+    float y[16];
+    if (kind != 2) {
+      // per-head RMSNorm over the 128 rows of the column, then rotary on pairs (r, r + 64)
+      float sq[16], tot[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) sq[j] = v[j] * v[j];
+      column_sums(sm, sub, lane, sq, tot);
+      const float gn = (kind == 0 ? o.qn : o.kn)[r];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) y[j] = v[j] * rsqrtf(tot[j] * (1.0f / BM) + o.eps) * gn;
+      if (r >= 64) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) sm.xch[j][r - 64] = y[j];
+      }
+      epi_bar();
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) y[j] = v[j];
+    }
+    if (kind == 2 || r < 64) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int col = c0 + j;
+        if (col >= cend) continue;
+        const int grow = o.row0 + col;
+        bf16 *dst;
+        if (kind == 0) {
+          dst = static_cast<bf16 *>(o.q_out) + ((size_t)grow * o.hq_row + head) * BM;
+        } else if (o.bk != nullptr) {
+          dst = static_cast<bf16 *>(kind == 1 ? o.bk : o.bv) + ((size_t)grow * o.hkv + kvh) * BM;
+        } else {
+          if (!o.wr[grow]) continue;
+          const int b = grow / o.R, pp = o.pos[grow];
+          const int page = o.page_table[(size_t)b * o.pages_per_seq + pp / o.page_size];
+          dst = static_cast<bf16 *>(o.pool) +
+                ((((size_t)page * 2 + (kind == 1 ? 0 : 1)) * o.hkv + kvh) * o.page_size + pp % o.page_size) * BM;
+        }
+        if (kind == 2) {
+          dst[r] = __float2bfloat16_rn(y[j]);
+        } else {
+          const float2 cs = o.rope[(size_t)o.pos[grow] * (BM / 2) + r];
+          const float x1 = y[j], x2 = sm.xch[j][r];
+          dst[r] = __float2bfloat16_rn(x1 * cs.x - x2 * cs.y);
+          dst[r + 64] = __float2bfloat16_rn(x2 * cs.x + x1 * cs.y);
+        }
+      }
+    }
+    if (kind != 2) epi_bar();  // xch is rewritten by the next chunk
   } else if constexpr (EP == EP_SWIGLU) {
     // rows 0..63 of the tile are gate features 64t.., rows 64..127 the matching up features
     if (r >= 64) {
@@ -276,6 +362,15 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
     pdl_wait();
+    if (p.ep.in_ss) {
+      // the input rows' RMSNorm, folded into a per-column scale of the product
+      for (int c = r; c < p.M; c += BM) {
+        float acc = 0.f;
+        for (int i = 0; i < p.ep.in_ss_n; ++i) acc += __ldcg(p.ep.in_ss + (size_t)i * p.ep.ld_ss + c);
+        sm.col_scale[c] = rsqrtf(acc * p.ep.in_inv_d + p.ep.in_eps);
+      }
+      epi_bar();
+    }
     // token columns this CTA finishes after the split-K reduction (multiple of 4)
     const int w4 = ((p.npad + 4 * p.P - 1) / (4 * p.P)) * 4;
     const int s0 = min(rank * w4, p.npad), s1 = min(min((rank + 1) * w4, p.npad), p.M);
@@ -333,16 +428,26 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
           for (int c0 = s0; c0 < s1; c0 += 16) {
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
-            for (int pr = 0; pr < p.P; ++pr) {  // fixed rank order: deterministic sum
-              const uint32_t base = mapa(my_row, (uint32_t)pr);
+            // peers in groups of four, fixed rank order (deterministic); a group's remote
+            // loads are all in flight together
+            for (int g0 = 0; g0 < p.P; g0 += 4) {
+              float4 x[4][4];
 #pragma unroll
-              for (int q4 = 0; q4 < 4; ++q4) {
-                if (c0 + 4 * q4 < s1) {
-                  const float4 x = ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4);
-                  v[4 * q4] += x.x;
-                  v[4 * q4 + 1] += x.y;
-                  v[4 * q4 + 2] += x.z;
-                  v[4 * q4 + 3] += x.w;
+              for (int gi = 0; gi < 4; ++gi) {
+                const uint32_t base = mapa(my_row, (uint32_t)min(g0 + gi, p.P - 1));
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                  x[gi][q4] = (g0 + gi < p.P && c0 + 4 * q4 < s1) ? ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4)
+                                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+              }
+#pragma unroll
+              for (int gi = 0; gi < 4; ++gi) {
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                  v[4 * q4] += x[gi][q4].x;
+                  v[4 * q4 + 1] += x[gi][q4].y;
+                  v[4 * q4 + 2] += x[gi][q4].z;
+                  v[4 * q4 + 3] += x[gi][q4].w;
                 }
               }
             }
@@ -601,6 +706,11 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
       ep.part_val += (size_t)m0 * ep.n_tiles;
       ep.part_idx += (size_t)m0 * ep.n_tiles;
     }
+    if (ep.in_ss) ep.in_ss += m0;
+    if (ep.out_ss) ep.out_ss += m0;
+    if (ep.out_xn) ep.out_xn = static_cast<bf16 *>(ep.out_xn) + (size_t)m0 * ep.ld_xn;
+    if (ep.out_stash) ep.out_stash = static_cast<bf16 *>(ep.out_stash) + (size_t)m0 * ep.ld_stash;
+    ep.qkv.row0 = m0;
     p.ep = ep;
     CUtensorMap mx;
     if (!tensor_map(&mx, static_cast<const bf16 *>(X) + (size_t)m0 * ldx, Mc, K, ldx, p.npad)) return cudaErrorInvalidValue;
@@ -611,6 +721,7 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
       case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s); break;
       case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s); break;
       case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s); break;
+      case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;
