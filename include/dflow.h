@@ -225,6 +225,24 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
                               const void *X, int32_t M, int32_t ldx, int32_t mode, void *out,
                               int32_t ldo, int32_t *status, void *stream);
 
+/* Greedy tokens without any device allocation (no counterpart in the paper:
+ * an integration aid for callers that cannot allocate device memory, e.g. code
+ * confined to a caller-owned memory pool or a plugin whose host owns all
+ * allocations).  tokens[r] = argmax_v hidden[r] . lm_head[v] (ties to the
+ * lowest id; -1 if a device error occurred), computed with the round's tensor-
+ * core LM-head kernels.
+ *   lm_head  bf16 [vocab][d], hidden bf16 [rows][d] (already final-normalised),
+ *   tokens   int32 [rows]; all device pointers owned by the caller.
+ * Limits: rows <= 64, vocab <= 262144 (else DFLOW_ERR_INVALID_ARG), d a
+ * multiple of 64, sm_103 devices only (else DFLOW_ERR_UNSUPPORTED).
+ * Scratch lives in a ~1 MiB array compiled into the library, held by every GPU
+ * that loads it until exit.  The first call on a device looks up that array's
+ * address (make it before any stream capture).  Calls share the array and it
+ * keeps the last call's contents; calls that overlap on the GPU race.  Calls
+ * no cudaMalloc/cudaFree and no allocating library routine. */
+dflow_status dflow_greedy_tokens_noalloc(const void *lm_head, int32_t vocab, int32_t d, const void *hidden,
+                                         int32_t rows, int32_t *tokens, void *stream);
+
 /* Waits for the recorded events, then fills out[DFLOW_PROF_N]. */
 dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out);
 /* Kernels launched by this handle since creation (always counted). */

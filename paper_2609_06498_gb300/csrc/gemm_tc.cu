@@ -518,13 +518,15 @@ cudaError_t launch_ep(const CUtensorMap &mw, const CUtensorMap &mx, const Params
 
 // clusters of P CTAs (with `smem` bytes each) that fit on the device at once
 template <int EP>
-int max_clusters(int P, size_t smem) {
+int max_clusters(int P, size_t smem, bool use_cache) {
   static std::mutex mu;
   static std::map<std::pair<int, size_t>, int> cache;
   std::lock_guard<std::mutex> lock(mu);
   auto key = std::make_pair(P, smem);
-  auto it = cache.find(key);
-  if (it != cache.end()) return it->second;
+  if (use_cache) {
+    auto it = cache.find(key);
+    if (it != cache.end()) return it->second;
+  }
   int n = 0;
   if (ensure_smem_attr<EP>() == cudaSuccess) {
     cudaLaunchConfig_t cfg = {};
@@ -541,7 +543,7 @@ int max_clusters(int P, size_t smem) {
     if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<EP>, &cfg) != cudaSuccess) n = 0;
   }
   cudaGetLastError();
-  cache.emplace(key, n);
+  if (use_cache) cache.emplace(key, n);
   return n;
 }
 
@@ -553,10 +555,10 @@ struct Choice {
 // split and cluster count minimising the k-blocks each CTA streams (plus a
 // small charge for the in-cluster reduction)
 template <int EP>
-Choice choose(int T, int kb, int npad, int sm_count) {
+Choice choose(int T, int kb, int npad, int sm_count, bool use_cache) {
   static std::mutex mu;
   static std::map<std::tuple<int, int, int>, Choice> cache;
-  {
+  if (use_cache) {
     std::lock_guard<std::mutex> lock(mu);
     auto it = cache.find(std::make_tuple(T, kb, npad));
     if (it != cache.end()) return it->second;
@@ -572,7 +574,7 @@ Choice choose(int T, int kb, int npad, int sm_count) {
     if (stages > 16) stages = 16;
     if (stages < 3) continue;
     const size_t smem = 1024 + (size_t)stages * stage_bytes + red_bytes + sizeof(Smem);
-    int Q = P == 1 ? sm_count : max_clusters<EP>(P, smem);
+    int Q = P == 1 ? sm_count : max_clusters<EP>(P, smem, use_cache);
     if (Q <= 0) continue;
     if (Q > T) Q = T;
     const long rounds = (T + Q - 1) / Q;
@@ -586,14 +588,16 @@ Choice choose(int T, int kb, int npad, int sm_count) {
       best.smem = smem;
     }
   }
-  std::lock_guard<std::mutex> lock(mu);
-  cache.emplace(std::make_tuple(T, kb, npad), best);
+  if (use_cache) {
+    std::lock_guard<std::mutex> lock(mu);
+    cache.emplace(std::make_tuple(T, kb, npad), best);
+  }
   return best;
 }
 
 template <int EP>
-cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_count, cudaStream_t s) {
-  const Choice c = choose<EP>(p.T, p.kb, p.npad, sm_count);
+cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_count, cudaStream_t s, bool use_cache) {
+  const Choice c = choose<EP>(p.T, p.kb, p.npad, sm_count, use_cache);
   if (c.P == 0) return cudaErrorInvalidValue;
   p.P = c.P;
   p.Q = c.Q;
@@ -634,15 +638,17 @@ struct MapKeyHash {
 };
 
 // bf16 row-major [rows][ld] matrix, tile box = 64 columns x box_rows rows, 128-byte swizzle
-bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows) {
+bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows, bool use_cache) {
   static std::mutex mu;
   static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
   const MapKey key{ptr, rows, cols, ld, box_rows};
   std::lock_guard<std::mutex> lock(mu);
-  auto it = cache.find(key);
-  if (it != cache.end()) {
-    *out = it->second;
-    return true;
+  if (use_cache) {
+    auto it = cache.find(key);
+    if (it != cache.end()) {
+      *out = it->second;
+      return true;
+    }
   }
   PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
   if (!enc) return false;
@@ -655,8 +661,10 @@ bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, i
           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return false;
-  if (cache.size() > 4096) cache.clear();
-  cache.emplace(key, m);
+  if (use_cache) {
+    if (cache.size() > 4096) cache.clear();
+    cache.emplace(key, m);
+  }
   *out = m;
   return true;
 }
@@ -682,9 +690,9 @@ cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s) {
 }
 
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
-                    const EpArgs &ep_in, int *status, cudaStream_t s) {
+                    const EpArgs &ep_in, int *status, cudaStream_t s, bool use_caches) {
   CUtensorMap mw;
-  if (!tensor_map(&mw, W, N, K, K, BM)) return cudaErrorInvalidValue;
+  if (!tensor_map(&mw, W, N, K, K, BM, use_caches)) return cudaErrorInvalidValue;
   for (int m0 = 0; m0 < M; m0 += MAX_NPAD) {
     const int Mc = M - m0 < MAX_NPAD ? M - m0 : MAX_NPAD;
     Params p{};
@@ -713,15 +721,16 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
     ep.qkv.row0 = m0;
     p.ep = ep;
     CUtensorMap mx;
-    if (!tensor_map(&mx, static_cast<const bf16 *>(X) + (size_t)m0 * ldx, Mc, K, ldx, p.npad)) return cudaErrorInvalidValue;
+    if (!tensor_map(&mx, static_cast<const bf16 *>(X) + (size_t)m0 * ldx, Mc, K, ldx, p.npad, use_caches))
+      return cudaErrorInvalidValue;
     cudaError_t e;
     switch (ep.mode) {
-      case EP_STORE_F32: e = run<EP_STORE_F32>(mw, mx, p, w.sm_count, s); break;
-      case EP_RESID: e = run<EP_RESID>(mw, mx, p, w.sm_count, s); break;
-      case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s); break;
-      case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s); break;
-      case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s); break;
-      case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s); break;
+      case EP_STORE_F32: e = run<EP_STORE_F32>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_RESID: e = run<EP_RESID>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s, use_caches); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;

@@ -8,7 +8,7 @@ namespace dflow {
 
 // 2D tensor map of a bf16 row-major [rows][ld] matrix, box 64 columns x box_rows
 // rows, 128-byte swizzle (cached by arguments).
-bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows);
+bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows, bool use_cache = true);
 
 // Scratch of the tensor-core GEMM inside the handle's workspace.
 struct TcWorkspace {
@@ -25,7 +25,9 @@ void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t row
 bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep);
 // Zero the counters once after the workspace is handed over.
 cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s);
+// use_caches = false: tensor maps are encoded on the stack and the launch plan
+// is recomputed, so the call touches no host heap
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M,
-                    int ldx, const EpArgs &ep, int *status, cudaStream_t s);
+                    int ldx, const EpArgs &ep, int *status, cudaStream_t s, bool use_caches = true);
 
 }  // namespace dflow
