@@ -157,11 +157,42 @@ def _stream(seed: int, name: str) -> np.random.Generator:
     return np.random.Generator(np.random.Philox(key=key))
 
 
-def normal(seed: int, name: str, shape, std: float = 0.02) -> np.ndarray:
-    """N(0, std^2) fp32 tensor, a pure function of (seed, name, shape)."""
+_CHUNK = 1 << 24
+_POOL = None
+
+
+def _pool():
+    global _POOL
+    if _POOL is None:
+        import concurrent.futures
+        import os
+        _POOL = concurrent.futures.ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1))
+    return _POOL
+
+
+def normal(seed: int, name: str, shape, std: float = 0.02, bf16: bool = False) -> np.ndarray:
+    """N(0, std^2) fp32 tensor, a pure function of (seed, name, shape).
+
+    Drawn in chunks of 2^24 values, chunk i from its own stream (seed, name#i),
+    so large tensors fill in parallel.  bf16=True rounds every value to the
+    nearest bf16 (kept in fp32 storage).
+    """
     n = int(np.prod(shape))
-    out = _stream(seed, name).standard_normal(n, dtype=np.float32)
-    out *= np.float32(std)
+    out = np.empty(n, np.float32)
+
+    def fill(i):
+        lo, hi = i * _CHUNK, min(n, (i + 1) * _CHUNK)
+        seg = out[lo:hi]
+        _stream(seed, f"{name}#{i}").standard_normal(hi - lo, dtype=np.float32, out=seg)
+        seg *= np.float32(std)
+        if bf16:
+            seg[:] = bf16_round(seg)
+
+    nchunks = (n + _CHUNK - 1) // _CHUNK
+    if nchunks <= 1:
+        fill(0) if n else None
+    else:
+        list(_pool().map(fill, range(nchunks)))
     return out.reshape(shape)
 
 
@@ -224,17 +255,21 @@ def weight(cfg: ModelConfig, name: str, seed: int = SEED_WEIGHTS,
                 w += 1.0
         else:
             w = np.zeros(shape, np.float32) if name == "ln_b" else np.ones(shape, np.float32)
+        if cfg.dtype == "bf16":
+            w = bf16_round(w)
     else:
-        w = normal(seed, name, shape, 0.02)
-    if cfg.dtype == "bf16":
-        w = bf16_round(w)
-    return w.astype(np.float32)
+        w = normal(seed, name, shape, 0.02, bf16=cfg.dtype == "bf16")
+    return w.astype(np.float32, copy=False)
 
 
 def weights(cfg: ModelConfig, seed: int = SEED_WEIGHTS, perturb_norms: bool = False,
             names: Optional[Iterable[str]] = None) -> Dict[str, np.ndarray]:
     names = list(tensor_shapes(cfg)) if names is None else list(names)
-    return {n: weight(cfg, n, seed, perturb_norms) for n in names}
+    big = [n for n in names if int(np.prod(tensor_shapes(cfg)[n])) > _CHUNK]
+    small = [n for n in names if n not in big]
+    out = {n: weight(cfg, n, seed, perturb_norms) for n in big}  # chunk-parallel inside
+    out.update(zip(small, _pool().map(lambda n: weight(cfg, n, seed, perturb_norms), small)))
+    return {n: out[n] for n in names}
 
 
 # --------------------------------------------------------------------------
@@ -312,8 +347,9 @@ def synthetic_state(cfg: ModelConfig, ctx_lens: Optional[np.ndarray] = None,
         for l in range(nl):
             for b in range(bs):
                 valid = int(lens[b]) - 1
-                arr[l, b, :valid] = normal(seed, f"st.{tag}{l}.{b}", (valid, hkv, hd), kv_std)
-        return bf16_round(arr) if cfg.dtype == "bf16" else arr
+                arr[l, b, :valid] = normal(seed, f"st.{tag}{l}.{b}", (valid, hkv, hd), kv_std,
+                                           bf16=cfg.dtype == "bf16")
+        return arr
 
     st["k"] = cache("k", cfg.n_layers)
     st["v"] = cache("v", cfg.n_layers)

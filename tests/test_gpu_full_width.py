@@ -1,0 +1,139 @@
+"""Parity at the real model widths of the four bf16 workloads (Qwen3 1.7B / 4B /
+8B shapes, batch 1-16, contexts 512-8192), one call at a time, and invariants
+of full-depth 8B rounds.
+
+The per-call tests run the kernels in exactly the launch configuration of the
+benchmark (every projection, attention and LM-head shape is per layer), on a
+copy of each model with 2 target layers and 1 draft layer so that the float64
+oracle finishes in seconds.  Caches are synthetic (seeded random K/V at the
+workload's context lengths)."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import Oracle
+from parity_util import assert_close, to_np, token_check, upload_state
+
+pytestmark = pytest.mark.gpu
+
+FULL = [synth.QWEN3_1P7B, synth.QWEN3_4B, synth.QWEN3_8B, synth.QWEN3_8B_KV]
+
+
+def reduced(cfg):
+    return cfg.replace(n_layers=2, draft_layers=1, feat_layers=(1, 2))
+
+
+@pytest.fixture(scope="module", params=FULL, ids=lambda c: c.name)
+def full(request):
+    from paper_2609_06498_gb300 import Engine, build, pack_weights
+    build.build()
+    cfg = reduced(request.param)
+    W = synth.weights(cfg, perturb_norms=True)
+    eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
+    o = Oracle(cfg, {k: v.astype(np.float64) for k, v in W.items()})
+    lens = synth.prompt_lengths(cfg) + 1
+    nc = np.array([[5, 0, 15, 9][b % 4] for b in range(cfg.batch)], np.int32)
+    ost = o.state_from_synthetic(synth.synthetic_state(cfg, ctx_lens=lens, n_carry=nc))
+    yield cfg, o, ost, eng
+    del eng
+    torch.cuda.empty_cache()
+
+
+def test_full_width_round_calls(full):
+    cfg, o, ost, eng = full
+    R, B, bs = cfg.rows, cfg.block, cfg.batch
+    st = eng.new_state(bs, page_seed=13)
+    upload_state(eng, st, ost)
+    ref = ost.copy()
+
+    # draft (Eq. 2, Eq. 4-5)
+    gblk = to_np(eng.draft_block(st))
+    oblk = np.zeros((bs, R), np.int32)
+    checked = 0
+    for b in range(bs):
+        oblk[b], lg, _ = o.draft_block(ref, b)
+        assert gblk[b, 0] == oblk[b, 0]
+        c, _ = token_check(gblk[b], oblk[b], lg, rows=range(1, R))
+        checked += c
+    assert checked >= bs * (B // 2)
+
+    # verify (Eq. 3 target side, Eq. 1) on the oracle's block
+    blk_t = torch.as_tensor(oblk).cuda()
+    g, feats, logits = eng.verify_block(st, blk_t, logits=True)
+    gg, gf, gl = to_np(g), to_np(feats), to_np(logits)
+    og = np.zeros((bs, R), np.int32)
+    of = np.zeros((bs, R, cfg.d))
+    for b in range(bs):
+        og[b], lg, of[b] = o.verify_block(ref, b, oblk[b])
+        assert_close(gl[b], lg, cfg, "verify logits")
+        assert_close(gf[b], of[b], cfg, "features")
+        token_check(gg[b], og[b], lg)
+        n = int(ref.seq_len[b])
+        k, v = st.read_cache(st.kv, b, n - 1 + R)
+        assert_close(to_np(k)[:, n - 1:], ref.k[:, b, n - 1:n - 1 + R], cfg, "block K")
+        assert_close(to_np(v)[:, n - 1:], ref.v[:, b, n - 1:n - 1 + R], cfg, "block V")
+
+    # accept/commit (Eq. 3) with the workload's forced schedule: bit exact
+    forced = synth.forced_schedule(cfg, 1)[0]
+    acc, comm = eng.accept_commit(st, blk_t, torch.as_tensor(og).cuda(), torch.as_tensor(forced).cuda())
+    oacc = np.zeros(bs, np.int32)
+    ocomm = np.zeros((bs, R), np.int32)
+    for b in range(bs):
+        oacc[b], ocomm[b] = o.accept_commit(ref, b, oblk[b], og[b], int(forced[b]))
+    assert np.array_equal(to_np(acc), oacc) and np.array_equal(to_np(comm), ocomm)
+    assert np.array_equal(to_np(st.seq_len), ref.seq_len)
+
+    # carry (Sec. 4.2) and context injection on the oracle's features
+    fin = torch.as_tensor(of).to(feats.dtype).cuda()
+    eng.carry_hidden(st, blk_t, fin, acc)
+    fin_np = to_np(fin)
+    for b in range(bs):
+        o.carry_hidden(ref, b, oblk[b], fin_np[b].astype(np.float64), int(oacc[b]))
+    assert np.array_equal(to_np(st.n_carry), ref.n_carry)
+    assert np.array_equal(to_np(st.boundary), ref.boundary)
+    gc = to_np(st.carry)
+    for b in range(bs):
+        nc = int(ref.n_carry[b])
+        assert np.array_equal(gc[b, :nc], fin_np[b, oacc[b] + 1:oacc[b] + 1 + nc])
+        n = int(ref.seq_len[b])
+        dk, dv = st.read_cache(st.draft_kv, b, n - 1)
+        lo = n - 2 - int(oacc[b])
+        assert_close(to_np(dk)[:, lo:], ref.dk[:, b, lo:n - 1], cfg, "ctx K append")
+        assert_close(to_np(dv)[:, lo:], ref.dv[:, b, lo:n - 1], cfg, "ctx V append")
+    assert eng.read_status(st) == 0
+
+
+def test_full_depth_8b_round_invariants():
+    """The benchmark workload itself (36 + 5 layers, prefill of 2048 tokens):
+    per-round properties that hold at any size, from the calls' own outputs."""
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = synth.QWEN3_8B
+    R, B = cfg.rows, cfg.block
+    eng = Engine(cfg, random_weights(cfg, seed=0), max_batch=1, max_ctx=cfg.max_ctx())
+    st = eng.new_state(1, page_seed=1)
+    eng.prefill(st, synth.prompts(cfg))
+    assert eng.read_status(st) == 0 and int(st.seq_len[0]) == cfg.prompt_len + 1
+    sched = synth.forced_schedule(cfg, 4)
+    for r in range(4):
+        n = int(st.seq_len[0])
+        blk = eng.draft_block(st)
+        g, feats, _ = eng.verify_block(st, blk)
+        forced = torch.as_tensor(sched[r]).cuda()
+        acc, comm = eng.accept_commit(st, blk, g, forced)
+        eng.carry_hidden(st, blk, feats, acc)
+        bk, gk, ck = to_np(blk)[0], to_np(g)[0], to_np(comm)[0]
+        a = int(acc[0])
+        assert a == int(sched[r][0])
+        assert bk[0] == to_np(st.tokens)[0, n - 1]  # row 0 is the anchor
+        assert list(ck[:a]) == list(bk[1:a + 1]) and ck[a] == gk[a] and (ck[a + 1:] == -1).all()
+        assert int(st.seq_len[0]) == n + a + 1
+        assert list(to_np(st.tokens)[0, n:n + a + 1]) == list(ck[:a + 1])
+        nc = max(0, B - a - 1)
+        assert int(st.n_carry[0]) == nc
+        assert np.array_equal(to_np(st.carry)[0, :nc], to_np(feats)[0, a + 1:a + 1 + nc])
+        bd = to_np(st.boundary)[0]
+        assert bd[0] == gk[a] and bd[1] == (bk[a + 1] if a < B else -1)
+        assert np.isfinite(to_np(feats)).all()
+    assert eng.read_status(st) == 0
