@@ -234,6 +234,30 @@ def run_reference(args):
 
 
 # --------------------------------------------------------------------------
+# multi-GPU replicas: each rank runs its own batch; the step time is the slowest
+# rank's and the throughput the sum of all ranks' committed tokens
+# --------------------------------------------------------------------------
+
+
+def reduce_scalar(x: float, op: str, device: str = "cpu") -> float:
+    """max or sum of a scalar over the ranks of the default process group."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def replica_throughput(committed_local: float, ms_local: float, world: int, device: str = "cpu"):
+    """(whole-job tokens/s, step time in ms) of `world` independent replicas."""
+    if world == 1:
+        return committed_local / (ms_local / 1e3), ms_local
+    tot = reduce_scalar(committed_local, "sum", device)
+    ms = reduce_scalar(ms_local, "max", device)
+    return tot / (ms / 1e3), ms
+
+
+# --------------------------------------------------------------------------
 # GPU arm
 # --------------------------------------------------------------------------
 
@@ -290,13 +314,6 @@ def main():
             dist.barrier()
         torch.cuda.synchronize()
 
-    def max_over_ranks(x: float) -> float:
-        if world == 1:
-            return x
-        t = torch.tensor([x], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
     if args.profile_only:
         # rounds inside a profiler range, for `ncu --profile-from-start off`
         torch.cuda.cudart().cudaProfilerStart()
@@ -326,8 +343,7 @@ def main():
     launches = eng.launch_count() - n0
     assert eng.read_status(st) == 0, "device status set during the timed leg"
     per = [ev[k].elapsed_time(ev[k + 1]) for k in range(K)]
-    total_ms = max_over_ranks(ev[0].elapsed_time(ev[K]))
-    value = committed * world / (total_ms / 1e3)
+    value, total_ms = replica_throughput(committed, ev[0].elapsed_time(ev[K]), world, "cuda")
 
     # ---- end-to-end leg: host buffers, H2D of the step's inputs and D2H of its result inside the region
     e2e = None
@@ -347,9 +363,9 @@ def main():
             h_comm[k].copy_(comm, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = max_over_ranks(e0.elapsed_time(e1))
+        e2e_value, _ = replica_throughput(committed, e0.elapsed_time(e1), world, "cuda")
         assert np.array_equal(h_acc.numpy(), sched[Wm:Wm + K]), "accept lengths differ from the schedule"
-        e2e = {"value": round(committed * world / (e2e_ms / 1e3), 2), "unit": "tokens/s",
+        e2e = {"value": round(e2e_value, 2), "unit": "tokens/s",
                "h2d_bytes_per_step": 4 * cfg.batch, "d2h_bytes_per_step": 4 * cfg.batch * (1 + cfg.rows)}
 
     # ---- profiled leg: per-launch events around the GEMMs (the dominant kernel)
