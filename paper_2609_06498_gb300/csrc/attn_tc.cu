@@ -19,6 +19,7 @@
 //     distributed shared memory, writing the final bf16 rows.  One launch per
 //     attention call, no global partials.
 #include <cuda.h>
+#include <stdlib.h>
 
 #include "dflow_internal.cuh"
 #include "gemm_tc.cuh"
@@ -427,6 +428,467 @@ cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnAr
   return cudaLaunchKernelEx(&cfg, k_attn_tc<HD, BLOCK>, tm, D, a, qgroups, status);
 }
 
+
+// ===========================================================================
+// tcgen05 variant (head_dim 128): queries are the MMA's M (padded to 128),
+// 64-key pages its N.  Warp 0 streams K/V pages (TMA), warp 1 issues
+// S = Q K^T and O += P V into TMEM, warps 2-5 own one query row per thread:
+// softmax straight out of TMEM (no shuffles), P to shared memory as the next
+// MMA's operand, lazy rescaling of the O row (only when the running max grows
+// by more than 2^8), zeroing of V rows past the context in a partial page.
+// ===========================================================================
+constexpr int T5_ROWS = 128;     // query rows per CTA (MMA M)
+constexpr int T5_STAGES = 5;     // K/V pages in flight
+constexpr int T5_SPLITS = 8;     // key splits = cluster size
+constexpr int T5_RPR = T5_ROWS / T5_SPLITS;
+constexpr float T5_TAU = 8.0f;   // rescale threshold, log2 units
+constexpr int T5_TMEM_COLS = 256;  // O: 128 columns, S: two buffers of 64
+
+struct T5Smem {
+  uint64_t kv_full[T5_STAGES], kv_empty[T5_STAGES], s_full[2], s_free[2], p_ready, pv_done, q_ready, drain;
+  uint32_t tmem;
+  float m[T5_ROWS], l[T5_ROWS], coef[T5_RPR * T5_SPLITS];
+};
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+      "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const float *v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+      "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+// the hardware base-2 exponential (approximate, flushes subnormals; 2^-inf = 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+// MN-major operand (row = k index, 64 contiguous n per 128-byte row), 128-byte
+// swizzle: 64-element n blocks `lbo` bytes apart, 8-row k groups 1024 bytes apart
+__device__ __forceinline__ uint64_t smem_desc_mn(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFF) >> 4);
+  d |= (uint64_t)(lbo >> 4) << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+template <bool BLOCK>
+__global__ void __launch_bounds__(THREADS, 1)
+k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *status) {
+  pdl_entry();
+  if (*status) return;
+  constexpr int HD = 128, TILE = 64 * HD * 2;  // one K or V page tile: 16 KB
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
+  uint8_t *qs = base;                                   // [2 boxes][128 rows][128 B]
+  uint8_t *ring = qs + 2 * T5_ROWS * 128;               // [stage][K | V]
+  uint8_t *ps = ring + T5_STAGES * 2 * TILE;            // [128 rows][64 keys] bf16
+  T5Smem &sm = *reinterpret_cast<T5Smem *>(ps + T5_ROWS * 128);
+  float *o_sm = reinterpret_cast<float *>(ring);        // [128][128] fp32 after the key loop
+
+  const int kvh = blockIdx.x, b = blockIdx.y;
+  const int split = blockIdx.z % T5_SPLITS, qg = blockIdx.z / T5_SPLITS;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int G = D.hq / D.hkv, R = D.R, QR = R * G, row0 = qg * T5_ROWS;
+  const int n_keys = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;
+  const int n_tiles = (n_keys + 63) / 64;
+  const int t_lo = (int)((long long)split * n_tiles / T5_SPLITS);
+  const int t_hi = (int)((long long)(split + 1) * n_tiles / T5_SPLITS);
+  const int T = (t_hi - t_lo) + ((BLOCK && split == T5_SPLITS - 1) ? 1 : 0);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < T5_STAGES; ++s) {
+      mbar_init(&sm.kv_full[s], 1);
+      mbar_init(&sm.kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&sm.s_full[i], 1);
+      mbar_init(&sm.s_free[i], 4);
+    }
+    mbar_init(&sm.p_ready, 4);
+    mbar_init(&sm.pv_done, 1);
+    mbar_init(&sm.q_ready, 4);
+    mbar_init(&sm.drain, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
+                 "r"(T5_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem;
+  const uint32_t t_o = tmem, t_s = tmem + 128;
+
+  if (warp == 0) {
+    // ---------------- producer: K/V pages ----------------
+    const int *pt = a.page_table + (size_t)b * D.pages_per_seq;
+    const uint64_t pol = policy_evict_first();
+    int n_issued = 0, pg = 0;
+    for (int it = 0; it < T; ++it) {
+      const int stage = it % T5_STAGES;
+      const uint32_t ph = (it / T5_STAGES) & 1;
+      const int tile = t_lo + it;
+      if ((it & 31) == 0) {
+        // page ids of the next 32 tiles, one per lane, fetched together
+        const int t = tile + lane;
+        pg = t < t_hi ? pt[t] : 0;
+      }
+      const int page = __shfl_sync(0xffffffffu, pg, it & 31);
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&sm.kv_empty[stage], ph ^ 1) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) {
+        if (lane == 0) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+        break;
+      }
+      uint8_t *kt = ring + (size_t)stage * 2 * TILE, *vt = kt + TILE;
+      if (tile < t_hi) {
+        if (lane == 0) {
+          const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;
+          mbar_expect_tx(&sm.kv_full[stage], 2 * TILE);
+          tma_load_2d(kt, &tm, 0, rk, &sm.kv_full[stage], pol);
+          tma_load_2d(kt + 8192, &tm, 64, rk, &sm.kv_full[stage], pol);
+          tma_load_2d(vt, &tm, 0, rv, &sm.kv_full[stage], pol);
+          tma_load_2d(vt + 8192, &tm, 64, rv, &sm.kv_full[stage], pol);
+        }
+      } else {
+        // the block's own K/V rows (drafter mode), zero past row R
+        const bf16 *bk = static_cast<const bf16 *>(a.bk), *bv = static_cast<const bf16 *>(a.bv);
+        for (int e = lane; e < 64 * (HD / 8); e += 32) {
+          const int j = e / (HD / 8), c = e % (HD / 8);
+          uint4 kx = make_uint4(0, 0, 0, 0), vx = make_uint4(0, 0, 0, 0);
+          if (j < R) {
+            const size_t off = ((size_t)(b * R + j) * D.hkv + kvh) * HD + c * 8;
+            kx = *reinterpret_cast<const uint4 *>(bk + off);
+            vx = *reinterpret_cast<const uint4 *>(bv + off);
+          }
+          *reinterpret_cast<uint4 *>(kt + swz(j, c)) = kx;
+          *reinterpret_cast<uint4 *>(vt + swz(j, c)) = vx;
+        }
+        fence_async_smem();  // generic-proxy writes read by the tensor cores
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.kv_full[stage]);
+      }
+      n_issued = it + 1;
+    }
+    // every fill of the last T5_STAGES has landed before the CTA may exit
+    if (lane == 0)
+      for (int it = n_issued > T5_STAGES ? n_issued - T5_STAGES : 0; it < n_issued; ++it)
+        if (!mbar_wait(&sm.kv_full[it % T5_STAGES], (uint32_t)((it / T5_STAGES) & 1)))
+          set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      constexpr uint32_t ID_S = (1u << 4) | (1u << 7) | (1u << 10) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
+      constexpr uint32_t ID_PV =
+          (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+      bool ok = mbar_wait(&sm.q_ready, 0);
+      const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
+      auto pv = [&](int j) -> bool {
+        if (!mbar_wait(&sm.p_ready, (uint32_t)(j & 1))) return false;
+        tc_fence_after();
+        const uint32_t vt = smem_u32(ring + (size_t)(j % T5_STAGES) * 2 * TILE + TILE);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          mma_bf16(t_o, smem_desc(pa + kk * 32), smem_desc_mn(vt + kk * 2048, 8192), ID_PV, (j > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&sm.kv_empty[j % T5_STAGES]);
+        mma_commit(&sm.pv_done);
+        return true;
+      };
+      for (int i = 0; i < T && ok; ++i) {
+        const int stage = i % T5_STAGES, buf = i & 1;
+        if (!mbar_wait(&sm.kv_full[stage], (uint32_t)((i / T5_STAGES) & 1)) ||
+            !mbar_wait(&sm.s_free[buf], (uint32_t)(((i >> 1) & 1) ^ 1))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kt = smem_u32(ring + (size_t)stage * 2 * TILE);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const uint32_t off = (kk >> 2) * 8192 + (kk & 3) * 32;
+          mma_bf16(t_s + buf * 64, smem_desc(qa + (kk >> 2) * 16384 + (kk & 3) * 32), smem_desc(kt + off), ID_S,
+                   kk > 0 ? 1u : 0u);
+        }
+        mma_commit(&sm.s_full[buf]);
+        if (i > 0 && !pv(i - 1)) ok = false;
+      }
+      if (ok && T > 0) ok = pv(T - 1);
+      if (!ok) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+      mma_commit(&sm.drain);
+      if (!mbar_wait(&sm.drain, 0)) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- softmax warps: thread = query row ----------------
+    const int sub = warp & 3, row = sub * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(sub * 32) << 16;
+    const int qr = row0 + row;
+    const bool valid = qr < QR;
+    const int qpos = valid ? a.pos[b * R + qr / G] : -1;
+    {
+      // this row of Q into the two 64-dim boxes (128-byte swizzle)
+      const bf16 *q = static_cast<const bf16 *>(a.q);
+      uint4 v[16];
+      if (valid) {
+        const uint4 *src = reinterpret_cast<const uint4 *>(q + ((size_t)(b * R + qr / G) * D.hq + kvh * G + qr % G) * HD);
+#pragma unroll
+        for (int c = 0; c < 16; ++c) v[c] = __ldg(src + c);
+      } else {
+#pragma unroll
+        for (int c = 0; c < 16; ++c) v[c] = make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int c = 0; c < 16; ++c)
+        *reinterpret_cast<uint4 *>(qs + (c >> 3) * (T5_ROWS * 128) + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v[c];
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.q_ready);
+    }
+    // keys this row may see: pool keys [0, vis_pool) (causal: up to its own
+    // position), block rows [0, vis_blk); rows past the group see nothing
+    const bool live = valid && qpos >= 0;
+    const int vis_pool = !live ? 0 : (a.causal ? min(n_keys, qpos + 1) : n_keys);
+    const int vis_blk = live ? R : 0;
+    const float sl2 = 1.4426950408889634f * rsqrtf((float)HD);
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int i = 0; i < T; ++i) {
+      const int buf = i & 1, stage = i % T5_STAGES, tile = t_lo + i;
+      const bool blk = tile >= t_hi;
+      int w_ok = 1;
+      if (lane == 0) w_ok = mbar_wait(&sm.s_full[buf], (uint32_t)((i >> 1) & 1)) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w_ok, 0)) { ok = false; break; }
+      mbar_wait(&sm.s_full[buf], (uint32_t)((i >> 1) & 1));
+      tc_fence_after();
+      float s[64];
+      tmem_ld32(t_s + lane_off + buf * 64, s);
+      tmem_ld32(t_s + lane_off + buf * 64 + 32, s + 32);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.s_free[buf]);
+      // raw scores; only a tile that crosses this row's limit is masked
+      const int lim_t = blk ? vis_blk : vis_pool - tile * 64;
+      if (lim_t < 64) {
+#pragma unroll
+        for (int j = 0; j < 64; ++j) s[j] = j < lim_t ? s[j] : -INFINITY;
+      }
+      // row max in four independent chains; the positive scale commutes with max
+      float m4[4] = {s[0], s[1], s[2], s[3]};
+#pragma unroll
+      for (int j = 4; j < 64; j += 4) {
+        m4[0] = fmaxf(m4[0], s[j]);
+        m4[1] = fmaxf(m4[1], s[j + 1]);
+        m4[2] = fmaxf(m4[2], s[j + 2]);
+        m4[3] = fmaxf(m4[3], s[j + 3]);
+      }
+      const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
+      const bool need = mx > m_used + T5_TAU || (m_used == -INFINITY && mx > -INFINITY);
+      const float m_new = need ? mx : m_used;
+      if (i > 0) {
+        // O holds tiles < i, and the P buffer is free again
+        int pv_ok = 1;
+        if (lane == 0) pv_ok = mbar_wait(&sm.pv_done, (uint32_t)((i - 1) & 1)) ? 1 : 0;
+        if (!__shfl_sync(0xffffffffu, pv_ok, 0)) { ok = false; break; }
+        mbar_wait(&sm.pv_done, (uint32_t)((i - 1) & 1));
+        tc_fence_after();
+        if (__any_sync(0xffffffffu, need)) {
+          const float corr = need ? (m_used == -INFINITY ? 0.f : exp2f(m_used - m_new)) : 1.f;
+          float o[32];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            tmem_ld32(t_o + lane_off + c * 32, o);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) o[j] *= corr;
+            tmem_st32(t_o + lane_off + c * 32, o);
+          }
+          l *= corr;
+        }
+      }
+      m_used = m_new;
+      // P = 2^(s * scale - m) (bf16) into the 128-byte-swizzled operand tile;
+      // masked scores are -inf and give 0 (a row with nothing visible yet has
+      // only masked scores, so the offset does not matter there)
+      const float nm = m_used == -INFINITY ? 0.f : -m_used;
+      float l4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        float p[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          p[e] = ex2_approx(fmaf(s[c * 8 + e], sl2, nm));
+          l4[e & 3] += p[e];
+        }
+        uint4 u;
+        u.x = pack_bf16(p[0], p[1]);
+        u.y = pack_bf16(p[2], p[3]);
+        u.z = pack_bf16(p[4], p[5]);
+        u.w = pack_bf16(p[6], p[7]);
+        *reinterpret_cast<uint4 *>(ps + row * 128 + (((c) ^ (row & 7)) << 4)) = u;
+      }
+      l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
+      if (!blk && tile * 64 + 64 > n_keys) {
+        // V rows past the context: zero them so stale bytes never meet P = 0
+        uint8_t *vt = ring + (size_t)stage * 2 * TILE + TILE;
+        const int z0 = max(n_keys - tile * 64, 0);
+        for (int e = row; e < (64 - z0) * 16; e += T5_ROWS) {
+          const int j = z0 + e / 16, c = e % 16;
+          *reinterpret_cast<uint4 *>(vt + swz(j, c)) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.p_ready);
+    }
+    if (!ok && lane == 0) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+    // ---- this split's unnormalised O row, max and sum
+    float o[128];
+    if (ok && T > 0) {
+      int pv_ok = 1;
+      if (lane == 0) pv_ok = mbar_wait(&sm.pv_done, (uint32_t)((T - 1) & 1)) ? 1 : 0;
+      pv_ok = __shfl_sync(0xffffffffu, pv_ok, 0);
+      if (pv_ok) {
+        mbar_wait(&sm.pv_done, (uint32_t)((T - 1) & 1));
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(t_o + lane_off + c * 32, o + c * 32);
+      } else {
+        if (lane == 0) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+#pragma unroll
+        for (int j = 0; j < 128; ++j) o[j] = 0.f;
+        m_used = -INFINITY;
+        l = 0.f;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 128; ++j) o[j] = 0.f;
+    }
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // (B) every softmax warp has drained TMEM
+    // the ring is reused for O once every copy and MMA has finished: wait for (A)
+    __syncthreads();  // (A)
+    // 16-byte chunks of a row XOR-permuted by (row & 7): eight consecutive rows
+    // hit distinct banks
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      *reinterpret_cast<float4 *>(o_sm + row * HD + ((j ^ (row & 7)) << 2)) =
+          make_float4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+    sm.m[row] = m_used;
+    sm.l[row] = l;
+  }
+  if (warp < 2) __syncthreads();  // (A) for the producer and MMA warps
+
+  // ---- merge the splits of this cluster: CTA `split` finishes rows [r_lo, r_hi)
+  __syncthreads();
+  cluster_sync();
+  const int r_lo = split * T5_RPR;
+  if (threadIdx.x < T5_RPR) {
+    const int rr = r_lo + threadIdx.x;
+    float ms[T5_SPLITS], ls[T5_SPLITS], M = -INFINITY;
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp) {
+      ms[sp] = ld_dsmem_f32(mapa(smem_u32(sm.m + rr), (uint32_t)sp));
+      ls[sp] = ld_dsmem_f32(mapa(smem_u32(sm.l + rr), (uint32_t)sp));
+    }
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp) M = fmaxf(M, ms[sp]);
+    float L = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp) L += (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M) * ls[sp];
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp)
+      sm.coef[threadIdx.x * T5_SPLITS + sp] = (ms[sp] == -INFINITY || L <= 0.f) ? 0.f : exp2f(ms[sp] - M) / L;
+  }
+  __syncthreads();
+  bf16 *out = static_cast<bf16 *>(a.out);
+  for (int e = threadIdx.x; e < T5_RPR * (HD / 4); e += THREADS) {
+    const int rr = r_lo + e / (HD / 4), d4 = (e % (HD / 4)) * 4, q_r = row0 + rr;
+    if (q_r >= QR) continue;
+    float4 x[T5_SPLITS];
+    const int off = rr * HD + (((d4 >> 2) ^ (rr & 7)) << 2);
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp) x[sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + off), (uint32_t)sp));
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int sp = 0; sp < T5_SPLITS; ++sp) {
+      const float c = sm.coef[(rr - r_lo) * T5_SPLITS + sp];
+      acc.x += c * x[sp].x;
+      acc.y += c * x[sp].y;
+      acc.z += c * x[sp].z;
+      acc.w += c * x[sp].w;
+    }
+    const int i = q_r / G, head = kvh * G + q_r % G;
+    bf16 *dst = out + ((size_t)(b * R + i) * D.hq + head) * HD + d4;
+    *reinterpret_cast<__nv_bfloat162 *>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
+    *reinterpret_cast<__nv_bfloat162 *>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
+  }
+  cluster_sync();  // peers may still read this CTA's shared memory until here
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(T5_TMEM_COLS) : "memory");
+  }
+}
+
+template <bool BLOCK>
+cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
+                      cudaStream_t s) {
+  const size_t smem = 1024 + 2 * T5_ROWS * 128 + T5_STAGES * 2 * (64 * 128 * 2) + T5_ROWS * 128 + sizeof(T5Smem);
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_attn_t5<BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  const int G = D.hq / D.hkv;
+  const int qgroups = (D.R * G + T5_ROWS - 1) / T5_ROWS;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(D.hkv, batch, T5_SPLITS * qgroups);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = 1;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = T5_SPLITS;
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK>, tm, D, a, status);
+}
+
 }  // namespace
 
 bool attention_tc_supported(const Dims &D) {
@@ -440,6 +902,8 @@ cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *st
   const int rows = D.num_pages * 2 * D.hkv * D.page_size;
   if (!tensor_map(&tm, a.pool, rows, D.hd, D.hd, 64)) return cudaErrorInvalidValue;
   const bool block = !a.causal;
+  if (D.hd == 128 && getenv("DFLOW_MMA_SYNC_ATTENTION") == nullptr)
+    return block ? launch_t5<true>(tm, D, batch, a, status, s) : launch_t5<false>(tm, D, batch, a, status, s);
   if (D.hd == 128) return block ? launch<128, true>(tm, D, batch, a, status, s) : launch<128, false>(tm, D, batch, a, status, s);
   return block ? launch<64, true>(tm, D, batch, a, status, s) : launch<64, false>(tm, D, batch, a, status, s);
 }
