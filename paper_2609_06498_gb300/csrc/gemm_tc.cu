@@ -66,7 +66,20 @@ struct Smem {
   int ri[4][16];
   float ssred[4][16];
   float col_scale[MAX_NPAD];
+  long long qkv_base[MAX_NPAD];  // EP_QKV, paged pool: element offset of the column's K slot of kv head 0, or -1
+  int qkv_pos[MAX_NPAD];         // EP_QKV: position of the column's row
 };
+
+// epilogue inputs that do not depend on the product, loaded while the MMAs run
+struct EpPre {
+  float x[16];    // EP_RESID: residual stream values of this row's feature at the chunk's columns
+  float gain;     // EP_RESID: next RMSNorm gain of the feature (out_xn)
+  float2 cs[16];  // EP_QKV: rotary (cos, sin) of pair r at the chunk's columns' positions
+  float gn;       // EP_QKV: q or k RMSNorm gain of row r
+};
+
+// SiLU from the fast exponential and division intrinsics (the result is rounded to bf16)
+__device__ __forceinline__ float silu_fast(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
@@ -83,10 +96,32 @@ __device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const f
   epi_bar();
 }
 
+// prefetch of the inputs epilogue_chunk(t, c0, nc) will need
+template <int EP>
+__device__ __forceinline__ void epilogue_prefetch(const Params &p, const Smem &sm, int t, int r, int c0, int nc,
+                                                  EpPre &pre) {
+  const EpArgs &ep = p.ep;
+  const int n = t * BM + r, ncol = min(c0 + nc, p.M) - c0;
+  if constexpr (EP == EP_RESID) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+      pre.x[j] = (n < p.N && j < ncol) ? __ldcg(ep.out_f32 + (size_t)(c0 + j) * ep.ldo + n) : 0.f;
+    pre.gain = (ep.out_xn != nullptr && n < p.N) ? ep.out_gain[n] : 0.f;
+  } else if constexpr (EP == EP_QKV) {
+    const QkvOut &o = ep.qkv;
+    pre.gn = t < o.nq + o.hkv ? (t < o.nq ? o.qn : o.kn)[r] : 0.f;
+    if (t < o.nq + o.hkv && r < 64) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        pre.cs[j] = j < ncol ? o.rope[(size_t)sm.qkv_pos[c0 + j] * (BM / 2) + r] : make_float2(0.f, 0.f);
+    }
+  }
+}
+
 // epilogue on token columns c0 .. c0+nc-1 (nc <= 16) of tile t; v[j] = D[row r][c0+j]
 template <int EP>
 __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t, int r, int sub, int lane, int c0,
-                                               int nc, float *v) {
+                                               int nc, float *v, const EpPre &pre) {
   const int n = t * BM + r;
   const EpArgs &ep = p.ep;
   const int cend = min(c0 + nc, p.M);
@@ -102,33 +137,36 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
         if (col < cend) {
           if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
           if constexpr (EP == EP_SILU)
-            reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_f(v[j]));
+            reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_fast(v[j]));
         }
       }
     }
   } else if constexpr (EP == EP_RESID) {
     float x[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j)
-      x[j] = (n < p.N && c0 + j < cend) ? ep.out_f32[(size_t)(c0 + j) * ep.ldo + n] : 0.f;
+    const bool row_ok = n < p.N, has_xn = ep.out_xn != nullptr, has_stash = ep.out_stash != nullptr;
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
       const int col = c0 + j;
-      if (n < p.N && col < cend) {
-        x[j] += v[j];
+      x[j] = pre.x[j] + v[j];
+      if (row_ok && col < cend) {
         ep.out_f32[(size_t)col * ep.ldo + n] = x[j];
-        if (ep.out_xn)
-          reinterpret_cast<bf16 *>(ep.out_xn)[(size_t)col * ep.ld_xn + n] = __float2bfloat16_rn(x[j] * ep.out_gain[n]);
-        if (ep.out_stash)
-          reinterpret_cast<bf16 *>(ep.out_stash)[(size_t)col * ep.ld_stash + n] = __float2bfloat16_rn(x[j]);
+        if (has_xn) reinterpret_cast<bf16 *>(ep.out_xn)[(size_t)col * ep.ld_xn + n] = __float2bfloat16_rn(x[j] * pre.gain);
+        if (has_stash) reinterpret_cast<bf16 *>(ep.out_stash)[(size_t)col * ep.ld_stash + n] = __float2bfloat16_rn(x[j]);
+      } else {
+        x[j] = 0.f;
       }
     }
     if (ep.out_ss) {
-      float sq[16], tot[16];
+      // squared-norm partial of this tile's 128 features; thread r < 16 owns column c0 + r
 #pragma unroll
-      for (int j = 0; j < 16; ++j) sq[j] = x[j] * x[j];
-      column_sums(sm, sub, lane, sq, tot);
-      if (r < 16 && c0 + r < cend) ep.out_ss[(size_t)t * ep.ld_ss + c0 + r] = tot[r];
+      for (int j = 0; j < 16; ++j) {
+        const float tj = warp_sum(x[j] * x[j]);
+        if (lane == 0) sm.ssred[sub][j] = tj;
+      }
+      epi_bar();
+      if (r < 16 && c0 + r < cend)
+        ep.out_ss[(size_t)t * ep.ld_ss + c0 + r] = sm.ssred[0][r] + sm.ssred[1][r] + sm.ssred[2][r] + sm.ssred[3][r];
+      epi_bar();
     }
   } else if constexpr (EP == EP_QKV) {
     const QkvOut &o = ep.qkv;
@@ -142,7 +180,7 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
 #pragma unroll
       for (int j = 0; j < 16; ++j) sq[j] = v[j] * v[j];
       column_sums(sm, sub, lane, sq, tot);
-      const float gn = (kind == 0 ? o.qn : o.kn)[r];
+      const float gn = pre.gn;
 #pragma unroll
       for (int j = 0; j < 16; ++j) y[j] = v[j] * rsqrtf(tot[j] * (1.0f / BM) + o.eps) * gn;
       if (r >= 64) {
@@ -155,27 +193,28 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
       for (int j = 0; j < 16; ++j) y[j] = v[j];
     }
     if (kind == 2 || r < 64) {
+      // destinations: q rows, the drafter's block K/V, or the column's slot in the paged pool
+      const size_t kv_off = (size_t)((kind == 1 ? 0 : o.hkv) + kvh) * o.page_size * BM;
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int col = c0 + j;
-        if (col >= cend) continue;
         const int grow = o.row0 + col;
         bf16 *dst;
+        bool wr = col < cend;
         if (kind == 0) {
           dst = static_cast<bf16 *>(o.q_out) + ((size_t)grow * o.hq_row + head) * BM;
         } else if (o.bk != nullptr) {
           dst = static_cast<bf16 *>(kind == 1 ? o.bk : o.bv) + ((size_t)grow * o.hkv + kvh) * BM;
         } else {
-          if (!o.wr[grow]) continue;
-          const int b = grow / o.R, pp = o.pos[grow];
-          const int page = o.page_table[(size_t)b * o.pages_per_seq + pp / o.page_size];
-          dst = static_cast<bf16 *>(o.pool) +
-                ((((size_t)page * 2 + (kind == 1 ? 0 : 1)) * o.hkv + kvh) * o.page_size + pp % o.page_size) * BM;
+          const long long base = wr ? sm.qkv_base[col] : -1;
+          wr = base >= 0;
+          dst = static_cast<bf16 *>(o.pool) + (wr ? (size_t)base + kv_off : 0);
         }
+        if (!wr) continue;
         if (kind == 2) {
           dst[r] = __float2bfloat16_rn(y[j]);
         } else {
-          const float2 cs = o.rope[(size_t)o.pos[grow] * (BM / 2) + r];
+          const float2 cs = pre.cs[j];
           const float x1 = y[j], x2 = sm.xch[j][r];
           dst[r] = __float2bfloat16_rn(x1 * cs.x - x2 * cs.y);
           dst[r + 64] = __float2bfloat16_rn(x2 * cs.x + x1 * cs.y);
@@ -196,7 +235,7 @@ __device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t,
         const int col = c0 + j;
         if (col < cend)
           reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + t * 64 + r] =
-              __float2bfloat16_rn(silu_f(v[j]) * sm.xch[j][r]);
+              __float2bfloat16_rn(silu_fast(v[j]) * sm.xch[j][r]);
       }
     }
     epi_bar();
@@ -276,8 +315,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       const uint64_t pw = policy_evict_first(), px = policy_evict_last();
       int stage = 0;
       uint32_t ph = 0;
-      int issued_phase[16];
-      for (int s = 0; s < 16; ++s) issued_phase[s] = -1;
+      int n_issued = 0;  // (tile, k-block) units whose copies were started, in ring order
       bool ok = true;
       const int nk = kr1 - kr0;
       const int n_units = ((p.T - q + p.Q - 1) / p.Q) * nk;  // (tile, k-block) pairs of this CTA, in order
@@ -286,8 +324,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       for (int u = 0; u < pre; ++u) {
         mbar_expect_tx(&sm.full[u], stage_bytes);
         tma_load_2d(ring + (size_t)u * stage_bytes, &tmW, (kr0 + u % nk) * BK, (q + (u / nk) * p.Q) * BM, &sm.full[u], pw);
-        issued_phase[u] = 0;
       }
+      n_issued = pre;
       pdl_wait();
       for (int u = 0; u < pre; ++u)
         tma_load_2d(ring + (size_t)u * stage_bytes + A_BYTES, &tmX, (kr0 + u % nk) * BK, 0, &sm.full[u], px);
@@ -303,7 +341,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         mbar_expect_tx(&sm.full[stage], stage_bytes);
         tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
         tma_load_2d(a + A_BYTES, &tmX, k * BK, 0, &sm.full[stage], px);
-        issued_phase[stage] = (int)ph;
+        n_issued = u + 1;
         if (++stage == p.stages) {
           stage = 0;
           ph ^= 1;
@@ -313,9 +351,10 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
         atomicExch(&sm.abort, 1);
       }
-      // every copy this thread started has landed before the CTA may exit
-      for (int s = 0; s < p.stages; ++s)
-        if (issued_phase[s] >= 0 && !mbar_wait(&sm.full[s], (uint32_t)issued_phase[s]))
+      // every copy this thread started has landed before the CTA may exit: the
+      // last fill of each stage is one of the last `stages` units
+      for (int u = n_issued > p.stages ? n_issued - p.stages : 0; u < n_issued; ++u)
+        if (!mbar_wait(&sm.full[u % p.stages], (uint32_t)((u / p.stages) & 1)))
           set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
     }
   } else if (warp == 1) {
@@ -371,12 +410,30 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       }
       epi_bar();
     }
+    if constexpr (EP == EP_QKV) {
+      // per token column: position, and the paged-pool slot its K/V rows go to
+      const QkvOut &o = p.ep.qkv;
+      for (int c = r; c < p.M; c += BM) {
+        const int grow = o.row0 + c, pp = o.pos[grow];
+        long long base = -1;
+        if (o.bk == nullptr && o.wr[grow]) {
+          const int page = o.page_table[(size_t)(grow / o.R) * o.pages_per_seq + pp / o.page_size];
+          base = ((long long)page * 2 * o.hkv * o.page_size + pp % o.page_size) * BM;
+        }
+        sm.qkv_pos[c] = pp;
+        sm.qkv_base[c] = base;
+      }
+      epi_bar();
+    }
     // token columns this CTA finishes after the split-K reduction (multiple of 4)
-    const int w4 = ((p.npad + 4 * p.P - 1) / (4 * p.P)) * 4;
-    const int s0 = min(rank * w4, p.npad), s1 = min(min((rank + 1) * w4, p.npad), p.M);
+    const int w4 = ((p.M + 4 * p.P - 1) / (4 * p.P)) * 4;
+    const int s0 = min(rank * w4, p.M), s1 = min((rank + 1) * w4, p.M);
+    const int c_first = p.P == 1 ? 0 : s0;
     int i = 0;
     for (int t = q; t < p.T; t += p.Q, ++i) {
       const int buf = i & 1;
+      EpPre pre;
+      epilogue_prefetch<EP>(p, sm, t, r, c_first, p.P == 1 ? 16 : min(16, s1 - s0), pre);
       if (leader) {
         int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
         if (ok && p.P > 1 && i > 0) ok = mbar_wait_cluster(&sm.freeb, (i - 1) & 1) ? 1 : 0;
@@ -396,8 +453,9 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       float v[16];
       if (p.P == 1) {
         for (int c0 = 0; c0 < p.npad && c0 < p.M; c0 += 16) {
+          if (c0 > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
           tmem_ld16(acc_addr + c0, v);
-          epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v);
+          epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v, pre);
         }
         tc_fence_before();
         __syncwarp();
@@ -423,6 +481,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         __syncwarp();
         epi_bar();
         const bool ok = sm.flag != 0;
+        bool released = false;
         if (ok) {
           const uint32_t my_row = smem_u32(mine);
           for (int c0 = s0; c0 < s1; c0 += 16) {
@@ -451,13 +510,26 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
                 }
               }
             }
-            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, min(16, s1 - c0), v);
+            if (c0 + 16 >= s1) {
+              // the last remote reads of this tile are done: the peers may overwrite their
+              // partials.  Signalled before the epilogue's global stores, which a release
+              // arrive after them would have to wait for.
+              epi_bar();
+              if (leader)
+                for (int pr = 0; pr < p.P; ++pr)
+                  if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+              released = true;
+            }
+            if (c0 > s0) epilogue_prefetch<EP>(p, sm, t, r, c0, min(16, s1 - c0), pre);
+            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
           }
         }
-        epi_bar();  // this CTA has finished reading every peer's partial
-        if (leader)
-          for (int pr = 0; pr < p.P; ++pr)
-            if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+        if (!released) {
+          epi_bar();  // this CTA has finished reading every peer's partial
+          if (leader)
+            for (int pr = 0; pr < p.P; ++pr)
+              if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+        }
         if (!ok) {
           if (leader) {
             set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
