@@ -292,7 +292,8 @@ def main():
     st = eng.new_state(cfg.batch, page_seed=rank)
     prompts = synth.prompts(cfg)
     eng.prefill(st, prompts)
-    assert eng.read_status(st) == 0, "prefill failed"
+    st_code = eng.read_status(st)
+    assert st_code == 0, f"prefill failed: device status {st_code}"
     sched = synth.forced_schedule(cfg, n_rounds, seed=synth.SEED_SCHEDULE + rank)
     forced_dev = torch.as_tensor(sched).cuda()
     acc = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
@@ -341,7 +342,8 @@ def main():
             ev[k + 1].record(stream)
         torch.cuda.synchronize()
     launches = eng.launch_count() - n0
-    assert eng.read_status(st) == 0, "device status set during the timed leg"
+    st_code = eng.read_status(st)
+    assert st_code == 0, f"device status {st_code} set during the timed leg"
     per = [ev[k].elapsed_time(ev[k + 1]) for k in range(K)]
     value, total_ms = replica_throughput(committed, ev[0].elapsed_time(ev[K]), world, "cuda")
 

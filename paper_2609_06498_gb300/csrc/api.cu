@@ -435,6 +435,7 @@ struct dflow_handle {
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
   int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen;
   TcWorkspace tcw;
+  DepChain dep;  // completion counters between consecutive tensor-core launches
   // measurement
   uint64_t n_launch = 0;
   bool prof = false;
@@ -452,10 +453,12 @@ namespace {
     if (e_ != cudaSuccess) return DFLOW_ERR_CUDA;    \
   } while (0)
 
+// a launch outside the counting chain: the next counting launch waits for its grid
 #define KL(...)          \
   do {                   \
     __VA_ARGS__;         \
     ++k.h->n_launch;     \
+    k.h->dep.brk();      \
   } while (0)
 
 struct Call {
@@ -504,6 +507,7 @@ size_t layout(dflow_handle *h, char *base) {
   h->plen = (int *)take((size_t)c.max_batch * 4);
   h->kvlen = (int *)take((size_t)c.max_batch * 4);
   h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
+  h->dep.dev = (unsigned int *)take(kDepSlots * sizeof(unsigned int));
   const int max_n = std::max(std::max(D.vocab, 2 * D.inter), std::max(h->gld, D.d));
   tc_layout(h->tcw, base, off, h->sm_count, rm, (max_n + 127) / 128);
   return off;
@@ -561,7 +565,9 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
   const double es = h->esz;
   ProfScope ps(h, k.s, DFLOW_PROF_GEMM, es * N * K + es * M * K + ep_out_bytes(ep, M, N, h->esz), 2.0 * M * N * K);
   ++h->n_launch;
-  if (h->use_tc && tc_supports(N, K, M, ldx, ep)) return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s);
+  if (h->use_tc && tc_supports(N, K, M, ldx, ep))
+    return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
+  h->dep.brk();
   return gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, k.status, k.s);
 }
 
@@ -703,7 +709,7 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
   {
     ProfScope ps(h, k.s, DFLOW_PROF_ATTN, 0.0, 4.0 * rows * D.hq * D.hd);
     h->n_launch += 2;
-    if ((e = attention(h->dtype, D, batch, a, k.status_w, k.s))) return e;
+    if ((e = attention(h->dtype, D, batch, a, k.status_w, k.s, &h->dep))) return e;
   }
   if (h->fused) {
     if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, resid_norm(h, L.mlp_norm, nullptr)))) return e;
@@ -926,8 +932,28 @@ dflow_status check_call(dflow_handle *h, const dflow_state *st) {
   return DFLOW_OK;
 }
 
+// start of a call: its first counting launch waits for the previous grid; after a
+// failed call the counters are zeroed (a launch may have been counted but not run)
 Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
+  DepChain &d = h->dep;
+  if (d.dirty && d.dev != nullptr) {
+    if (cudaMemsetAsync(d.dev, 0, kDepSlots * sizeof(unsigned int), (cudaStream_t)stream) == cudaSuccess) {
+      for (int i = 0; i < kDepSlots; ++i) d.shadow[i] = 0;
+      d.next = 0;
+      d.dirty = false;
+    } else {
+      cudaGetLastError();
+      d.dev = nullptr;  // counting off for this handle: every launch waits for its predecessor's grid
+    }
+  }
+  d.brk();
   return Call{h, st->status, st->status, (cudaStream_t)stream};
+}
+
+// a failed call leaves the counters unknown
+dflow_status finish(dflow_handle *h, dflow_status r) {
+  if (r != DFLOW_OK) h->dep.dirty = true;
+  return r;
 }
 
 bool valid_layer(const dflow_layer_weights &L) {
@@ -1067,8 +1093,8 @@ dflow_status dflow_prefill(dflow_handle *h, dflow_state *st, const int32_t *prom
     if (len + 1 + h->R > h->cfg.max_ctx) return DFLOW_ERR_CAPACITY;
   }
   Call k = make_call(h, st, stream);
-  return h->dtype == DFLOW_BF16 ? do_prefill<bf16>(k, st, prompt, prompt_stride, prompt_len_host)
-                                : do_prefill<float>(k, st, prompt, prompt_stride, prompt_len_host);
+  return finish(h, h->dtype == DFLOW_BF16 ? do_prefill<bf16>(k, st, prompt, prompt_stride, prompt_len_host)
+                                          : do_prefill<float>(k, st, prompt, prompt_stride, prompt_len_host));
 }
 
 dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens, void *stream) {
@@ -1076,8 +1102,9 @@ dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_
   if (r) return r;
   if (!block_tokens) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return r;
-  return h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1) : do_draft<float>(k, st, block_tokens, 1);
+  if ((r = guard(k, st))) return finish(h, r);
+  return finish(h, h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1)
+                                          : do_draft<float>(k, st, block_tokens, 1));
 }
 
 dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
@@ -1086,9 +1113,9 @@ dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t 
   if (r) return r;
   if (!block_tokens || !target_argmax || !feats) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return r;
-  return h->dtype == DFLOW_BF16 ? do_verify<bf16>(k, st, block_tokens, target_argmax, feats, logits)
-                                : do_verify<float>(k, st, block_tokens, target_argmax, feats, logits);
+  if ((r = guard(k, st))) return finish(h, r);
+  return finish(h, h->dtype == DFLOW_BF16 ? do_verify<bf16>(k, st, block_tokens, target_argmax, feats, logits)
+                                          : do_verify<float>(k, st, block_tokens, target_argmax, feats, logits));
 }
 
 dflow_status dflow_accept_commit(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
@@ -1098,7 +1125,7 @@ dflow_status dflow_accept_commit(dflow_handle *h, dflow_state *st, const int32_t
   if (r) return r;
   if (!block_tokens || !target_argmax || !accept_len || !committed) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  return do_accept(k, st, block_tokens, target_argmax, forced_accept, accept_len, committed);
+  return finish(h, do_accept(k, st, block_tokens, target_argmax, forced_accept, accept_len, committed));
 }
 
 dflow_status dflow_carry_hidden(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,
@@ -1107,8 +1134,8 @@ dflow_status dflow_carry_hidden(dflow_handle *h, dflow_state *st, const int32_t 
   if (r) return r;
   if (!block_tokens || !feats || !accept_len) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  return h->dtype == DFLOW_BF16 ? do_carry<bf16>(k, st, block_tokens, feats, accept_len, 1)
-                                : do_carry<float>(k, st, block_tokens, feats, accept_len, 1);
+  return finish(h, h->dtype == DFLOW_BF16 ? do_carry<bf16>(k, st, block_tokens, feats, accept_len, 1)
+                                          : do_carry<float>(k, st, block_tokens, feats, accept_len, 1));
 }
 
 dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced_accept, int32_t *accept_len,
@@ -1117,17 +1144,17 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
   if (r) return r;
   if (!accept_len || !committed) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return r;
+  if ((r = guard(k, st))) return finish(h, r);
   if (h->dtype == DFLOW_BF16) {
-    if ((r = do_draft<bf16>(k, st, h->blk, relay))) return r;
-    if ((r = do_verify<bf16>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
-    if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return r;
-    return do_carry<bf16>(k, st, h->blk, h->feats, accept_len, relay);
+    if ((r = do_draft<bf16>(k, st, h->blk, relay))) return finish(h, r);
+    if ((r = do_verify<bf16>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
+    if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
+    return finish(h, do_carry<bf16>(k, st, h->blk, h->feats, accept_len, relay));
   }
-  if ((r = do_draft<float>(k, st, h->blk, relay))) return r;
-  if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
-  if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return r;
-  return do_carry<float>(k, st, h->blk, h->feats, accept_len, relay);
+  if ((r = do_draft<float>(k, st, h->blk, relay))) return finish(h, r);
+  if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
+  if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
+  return finish(h, do_carry<float>(k, st, h->blk, h->feats, accept_len, relay));
 }
 
 dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable) {

@@ -179,9 +179,11 @@ cudaError_t launch(const Dims &D, int batch, const AttnArgs &a, const int *statu
 
 }  // namespace
 
-cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s) {
+cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s,
+                      DepChain *chain) {
   if (dtype == DFLOW_BF16 && attention_tc_supported(D) && getenv("DFLOW_SIMT_ATTENTION") == nullptr)
-    return attention_tc(D, batch, a, status, s);
+    return attention_tc(D, batch, a, status, s, chain);
+  if (chain) chain->brk();
   if (D.hd == 128)
     return dtype == DFLOW_BF16 ? launch<bf16, 128>(D, batch, a, status, s)
                                : launch<float, 128>(D, batch, a, status, s);

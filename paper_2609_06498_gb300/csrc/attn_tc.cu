@@ -431,23 +431,30 @@ cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnAr
 
 // ===========================================================================
 // tcgen05 variant (head_dim 128): queries are the MMA's M (padded to 128),
-// 64-key pages its N.  Warp 0 streams K/V pages (TMA), warp 1 issues
-// S = Q K^T and O += P V into TMEM, warps 2-5 own one query row per thread:
-// softmax straight out of TMEM (no shuffles), P to shared memory as the next
-// MMA's operand, lazy rescaling of the O row (only when the running max grows
-// by more than 2^8), zeroing of V rows past the context in a partial page.
+// 64-key pages its N.  Warp 0 streams K/V pages (TMA; split s of the cluster
+// takes pages s, s + 8, ...) and the query rows (two 3D TMA boxes that land in
+// MMA row order), issuing the first copies right after the dependency wait;
+// warp 1 issues S = Q K^T and O += P V into TMEM; warps 2-5 own one query row
+// per thread: softmax straight out of TMEM (no shuffles), P to one of two
+// shared-memory tiles (so the next page's softmax overlaps this page's P V),
+// lazy rescaling of the O row (only when the running max grows by more than
+// 2^8), zeroing of V rows past the context in a partial page.  The splits
+// merge their (O, max, sum) through distributed shared memory.
 // ===========================================================================
 constexpr int T5_ROWS = 128;     // query rows per CTA (MMA M)
-constexpr int T5_STAGES = 5;     // K/V pages in flight
-constexpr int T5_SPLITS = 8;     // key splits = cluster size
-constexpr int T5_RPR = T5_ROWS / T5_SPLITS;
+constexpr int T5_STAGES = 4;     // K/V pages in flight
+constexpr int T5_SPLITS = 8;     // key splits = cluster size; split s takes pages s, s + 8, ...
 constexpr float T5_TAU = 8.0f;   // rescale threshold, log2 units
 constexpr int T5_TMEM_COLS = 256;  // O: 128 columns, S: two buffers of 64
 
 struct T5Smem {
-  uint64_t kv_full[T5_STAGES], kv_empty[T5_STAGES], s_full[2], s_free[2], p_ready, pv_done, q_ready, drain;
+  // two P buffers, each with its own ready / consumed barrier: a buffer is
+  // rewritten only after its previous P V is done, so neither barrier can run
+  // two phases ahead of its waiter
+  uint64_t kv_full[T5_STAGES], kv_empty[T5_STAGES], s_full[2], s_free[2], p_ready[2], pv_done[2], q_full, drain;
   uint32_t tmem;
-  float m[T5_ROWS], l[T5_ROWS], coef[T5_RPR * T5_SPLITS];
+  int n_keys;
+  float m[T5_ROWS], l[T5_ROWS];
 };
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float *v) {
@@ -498,71 +505,121 @@ __device__ __forceinline__ uint64_t smem_desc_mn(uint32_t saddr, uint32_t lbo) {
   d |= (uint64_t)2 << 61;
   return d;
 }
+// pages of split s: s, s + T5_SPLITS, ...; the ones below n_tiles hold keys
+__device__ __forceinline__ int t5_pool_tiles(int n_tiles, int split) {
+  return n_tiles > split ? (n_tiles - 1 - split) / T5_SPLITS + 1 : 0;
+}
 
+// q_tma: the CTA's query rows arrive as two boxes of the 3D map tq over
+// [rows][hq][128] (64 dims x G heads x R rows); else each softmax thread loads its row
 template <bool BLOCK>
 __global__ void __launch_bounds__(THREADS, 1)
-k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *status) {
-  pdl_entry();
-  if (*status) return;
+k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tq, Dims D, AttnArgs a,
+          int q_tma, int *status) {
+  // runs even after an earlier error (every wait is bounded): the CTAs of a
+  // cluster must not disagree on whether to take part in its barriers
+  pdl_trigger();
   constexpr int HD = 128, TILE = 64 * HD * 2;  // one K or V page tile: 16 KB
+  constexpr int PBUF = T5_ROWS * 128;          // one P tile: [128 rows][64 keys] bf16
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
-  uint8_t *qs = base;                                   // [2 boxes][128 rows][128 B]
-  uint8_t *ring = qs + 2 * T5_ROWS * 128;               // [stage][K | V]
-  uint8_t *ps = ring + T5_STAGES * 2 * TILE;            // [128 rows][64 keys] bf16
-  T5Smem &sm = *reinterpret_cast<T5Smem *>(ps + T5_ROWS * 128);
-  float *o_sm = reinterpret_cast<float *>(ring);        // [128][128] fp32 after the key loop
+  uint8_t *qs = base;                          // [2 boxes][128 rows][128 B]
+  uint8_t *ring = qs + 2 * T5_ROWS * 128;      // [stage][K | V]
+  uint8_t *ps = ring + T5_STAGES * 2 * TILE;   // [2][P tile]
+  T5Smem &sm = *reinterpret_cast<T5Smem *>(ps + 2 * PBUF);
+  float *o_sm = reinterpret_cast<float *>(ring);  // [128][128] fp32 after the key loop
 
   const int kvh = blockIdx.x, b = blockIdx.y;
   const int split = blockIdx.z % T5_SPLITS, qg = blockIdx.z / T5_SPLITS;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = D.hq / D.hkv, R = D.R, QR = R * G, row0 = qg * T5_ROWS;
-  const int n_keys = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;
-  const int n_tiles = (n_keys + 63) / 64;
-  const int t_lo = (int)((long long)split * n_tiles / T5_SPLITS);
-  const int t_hi = (int)((long long)(split + 1) * n_tiles / T5_SPLITS);
-  const int T = (t_hi - t_lo) + ((BLOCK && split == T5_SPLITS - 1) ? 1 : 0);
+  const int *pt = a.page_table + (size_t)b * D.pages_per_seq;
+  const uint64_t pol = policy_evict_first();
 
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < T5_STAGES; ++s) {
-      mbar_init(&sm.kv_full[s], 1);
-      mbar_init(&sm.kv_empty[s], 1);
+  // warp 0: the K/V (and Q) copies that do not wait for a free stage start right
+  // after the dependency wait, before the CTA-wide barrier
+  int pg = 0, n_pre = 0, nk = 0;
+  if (warp == 0) {
+    // page ids of this split's first 32 pages: the page table is the caller's
+    // and does not change during a call
+    const int t = split + T5_SPLITS * lane;
+    pg = t < D.pages_per_seq ? __ldg(pt + t) : 0;
+    if (lane == 0) {
+      prefetch_tensormap(&tm);
+      if (q_tma) prefetch_tensormap(&tq);
+      for (int s = 0; s < T5_STAGES; ++s) {
+        mbar_init(&sm.kv_full[s], 1);
+        mbar_init(&sm.kv_empty[s], 1);
+      }
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&sm.s_full[i], 1);
+        mbar_init(&sm.s_free[i], 4);
+        mbar_init(&sm.pv_done[i], 1);
+        mbar_init(&sm.p_ready[i], 4);
+      }
+      mbar_init(&sm.q_full, q_tma ? 1 : 4);
+      mbar_init(&sm.drain, 1);
+      asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+      dep_wait(a.dep, status);
+      nk = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;  // consumed after the first copies are issued
+      if (a.dep.wait) fence_proxy_async_global();  // Q and K/V rows just written by the projection, read by TMA
+      if (q_tma) {
+        const uint32_t qbytes = (uint32_t)(R * G * 128);
+        mbar_expect_tx(&sm.q_full, 2 * qbytes);
+        tma_load_3d(qs, &tq, 0, kvh * G, b * R, &sm.q_full);
+        tma_load_3d(qs + T5_ROWS * 128, &tq, 64, kvh * G, b * R, &sm.q_full);
+      }
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&sm.s_full[i], 1);
-      mbar_init(&sm.s_free[i], 4);
+    __syncwarp();  // the other lanes read the previous launches' outputs after lane 0's wait
+    if constexpr (BLOCK) {
+      // drafter: the block's own tile follows the pool pages, so the key count
+      // decides the first fills
+      nk = __shfl_sync(0xffffffffu, nk, 0);
+      n_pre = min(t5_pool_tiles((nk + 63) / 64, split), T5_STAGES);
+    } else {
+      // the split's first pages go out before the key count is known: a page
+      // past the context is loaded but never consumed (its copy is still
+      // drained), a page id past the pool reads as fill
+      n_pre = min(T5_STAGES, (D.pages_per_seq - split + T5_SPLITS - 1) / T5_SPLITS);
     }
-    mbar_init(&sm.p_ready, 4);
-    mbar_init(&sm.pv_done, 1);
-    mbar_init(&sm.q_ready, 4);
-    mbar_init(&sm.drain, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (warp == 1) {
+    for (int it = 0; it < n_pre; ++it) {
+      const int page = __shfl_sync(0xffffffffu, pg, it);
+      if (lane == 0) {
+        uint8_t *kt = ring + (size_t)it * 2 * TILE, *vt = kt + TILE;
+        const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;
+        mbar_expect_tx(&sm.kv_full[it], 2 * TILE);
+        tma_load_2d(kt, &tm, 0, rk, &sm.kv_full[it], pol);
+        tma_load_2d(kt + 8192, &tm, 64, rk, &sm.kv_full[it], pol);
+        tma_load_2d(vt, &tm, 0, rv, &sm.kv_full[it], pol);
+        tma_load_2d(vt + 8192, &tm, 64, rv, &sm.kv_full[it], pol);
+      }
+    }
+    if (lane == 0) sm.n_keys = nk;
+  } else if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
                  "r"(T5_TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  __syncthreads();
+  __syncthreads();  // barriers, TMEM and the key count are in place; thread 0's wait orders every later read
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
   const uint32_t t_o = tmem, t_s = tmem + 128;
+  const int n_keys = sm.n_keys;
+  const int n_tiles = (n_keys + 63) / 64;
+  const int Tp = t5_pool_tiles(n_tiles, split);
+  const int T = Tp + ((BLOCK && split == T5_SPLITS - 1) ? 1 : 0);
 
   if (warp == 0) {
-    // ---------------- producer: K/V pages ----------------
-    const int *pt = a.page_table + (size_t)b * D.pages_per_seq;
-    const uint64_t pol = policy_evict_first();
-    int n_issued = 0, pg = 0;
-    for (int it = 0; it < T; ++it) {
+    // ---------------- producer: the remaining K/V pages ----------------
+    int n_issued = n_pre;
+    for (int it = n_pre; it < T; ++it) {
       const int stage = it % T5_STAGES;
       const uint32_t ph = (it / T5_STAGES) & 1;
-      const int tile = t_lo + it;
       if ((it & 31) == 0) {
-        // page ids of the next 32 tiles, one per lane, fetched together
-        const int t = tile + lane;
-        pg = t < t_hi ? pt[t] : 0;
+        const int t = split + T5_SPLITS * (it + lane);
+        pg = (it + lane < Tp) ? pt[t] : 0;
       }
       const int page = __shfl_sync(0xffffffffu, pg, it & 31);
       int ok = 1;
@@ -572,7 +629,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
         break;
       }
       uint8_t *kt = ring + (size_t)stage * 2 * TILE, *vt = kt + TILE;
-      if (tile < t_hi) {
+      if (it < Tp) {
         if (lane == 0) {
           const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;
           mbar_expect_tx(&sm.kv_full[stage], 2 * TILE);
@@ -602,10 +659,12 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
       n_issued = it + 1;
     }
     // every fill of the last T5_STAGES has landed before the CTA may exit
-    if (lane == 0)
+    if (lane == 0) {
       for (int it = n_issued > T5_STAGES ? n_issued - T5_STAGES : 0; it < n_issued; ++it)
         if (!mbar_wait(&sm.kv_full[it % T5_STAGES], (uint32_t)((it / T5_STAGES) & 1)))
           set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+      if (q_tma && !mbar_wait(&sm.q_full, 0)) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
+    }
     __syncwarp();
   } else if (warp == 1) {
     // ---------------- MMA issuer ----------------
@@ -613,17 +672,18 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
       constexpr uint32_t ID_S = (1u << 4) | (1u << 7) | (1u << 10) | ((64u >> 3) << 17) | ((128u >> 4) << 24);
       constexpr uint32_t ID_PV =
           (1u << 4) | (1u << 7) | (1u << 10) | (1u << 16) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
-      bool ok = mbar_wait(&sm.q_ready, 0);
+      bool ok = mbar_wait(&sm.q_full, 0);
       const uint32_t qa = smem_u32(qs), pa = smem_u32(ps);
       auto pv = [&](int j) -> bool {
-        if (!mbar_wait(&sm.p_ready, (uint32_t)(j & 1))) return false;
+        if (!mbar_wait(&sm.p_ready[j & 1], (uint32_t)((j >> 1) & 1))) return false;
         tc_fence_after();
         const uint32_t vt = smem_u32(ring + (size_t)(j % T5_STAGES) * 2 * TILE + TILE);
+        const uint32_t pj = pa + (uint32_t)(j & 1) * PBUF;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
-          mma_bf16(t_o, smem_desc(pa + kk * 32), smem_desc_mn(vt + kk * 2048, 8192), ID_PV, (j > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16(t_o, smem_desc(pj + kk * 32), smem_desc_mn(vt + kk * 2048, 8192), ID_PV, (j > 0 || kk > 0) ? 1u : 0u);
         mma_commit(&sm.kv_empty[j % T5_STAGES]);
-        mma_commit(&sm.pv_done);
+        mma_commit(&sm.pv_done[j & 1]);
         return true;
       };
       for (int i = 0; i < T && ok; ++i) {
@@ -657,7 +717,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
     const int qr = row0 + row;
     const bool valid = qr < QR;
     const int qpos = valid ? a.pos[b * R + qr / G] : -1;
-    {
+    if (!q_tma) {
       // this row of Q into the two 64-dim boxes (128-byte swizzle)
       const bf16 *q = static_cast<const bf16 *>(a.q);
       uint4 v[16];
@@ -674,7 +734,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
         *reinterpret_cast<uint4 *>(qs + (c >> 3) * (T5_ROWS * 128) + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = v[c];
       fence_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.q_ready);
+      if (lane == 0) mbar_arrive(&sm.q_full);
     }
     // keys this row may see: pool keys [0, vis_pool) (causal: up to its own
     // position), block rows [0, vis_blk); rows past the group see nothing
@@ -684,13 +744,18 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
     const float sl2 = 1.4426950408889634f * rsqrtf((float)HD);
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int i = 0; i < T; ++i) {
-      const int buf = i & 1, stage = i % T5_STAGES, tile = t_lo + i;
-      const bool blk = tile >= t_hi;
+    auto wait_all = [&](uint64_t *bar, uint32_t parity) -> bool {
       int w_ok = 1;
-      if (lane == 0) w_ok = mbar_wait(&sm.s_full[buf], (uint32_t)((i >> 1) & 1)) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w_ok, 0)) { ok = false; break; }
-      mbar_wait(&sm.s_full[buf], (uint32_t)((i >> 1) & 1));
+      if (lane == 0) w_ok = mbar_wait(bar, parity) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w_ok, 0)) return false;
+      mbar_wait(bar, parity);  // completed: every lane observes it
+      return true;
+    };
+    for (int i = 0; i < T; ++i) {
+      const int buf = i & 1, stage = i % T5_STAGES;
+      const bool blk = i >= Tp;
+      const int tile = split + T5_SPLITS * i;
+      if (!wait_all(&sm.s_full[buf], (uint32_t)((i >> 1) & 1))) { ok = false; break; }
       tc_fence_after();
       float s[64];
       tmem_ld32(t_s + lane_off + buf * 64, s);
@@ -716,31 +781,29 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
       const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * sl2;
       const bool need = mx > m_used + T5_TAU || (m_used == -INFINITY && mx > -INFINITY);
       const float m_new = need ? mx : m_used;
-      if (i > 0) {
-        // O holds tiles < i, and the P buffer is free again
-        int pv_ok = 1;
-        if (lane == 0) pv_ok = mbar_wait(&sm.pv_done, (uint32_t)((i - 1) & 1)) ? 1 : 0;
-        if (!__shfl_sync(0xffffffffu, pv_ok, 0)) { ok = false; break; }
-        mbar_wait(&sm.pv_done, (uint32_t)((i - 1) & 1));
+      if (i > 0 && __any_sync(0xffffffffu, need)) {
+        // rescale O: it must hold tiles < i (the P V of tile i - 1 is done)
+        if (!wait_all(&sm.pv_done[(i - 1) & 1], (uint32_t)(((i - 1) >> 1) & 1))) { ok = false; break; }
         tc_fence_after();
-        if (__any_sync(0xffffffffu, need)) {
-          const float corr = need ? (m_used == -INFINITY ? 0.f : exp2f(m_used - m_new)) : 1.f;
-          float o[32];
+        const float corr = need ? (m_used == -INFINITY ? 0.f : exp2f(m_used - m_new)) : 1.f;
+        float o[32];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            tmem_ld32(t_o + lane_off + c * 32, o);
+        for (int c = 0; c < 4; ++c) {
+          tmem_ld32(t_o + lane_off + c * 32, o);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) o[j] *= corr;
-            tmem_st32(t_o + lane_off + c * 32, o);
-          }
-          l *= corr;
+          for (int j = 0; j < 32; ++j) o[j] *= corr;
+          tmem_st32(t_o + lane_off + c * 32, o);
         }
+        l *= corr;
       }
       m_used = m_new;
+      // the P buffer of tile i - 2 is free once its P V is done
+      if (i > 1 && !wait_all(&sm.pv_done[buf], (uint32_t)(((i - 2) >> 1) & 1))) { ok = false; break; }
       // P = 2^(s * scale - m) (bf16) into the 128-byte-swizzled operand tile;
       // masked scores are -inf and give 0 (a row with nothing visible yet has
       // only masked scores, so the offset does not matter there)
       const float nm = m_used == -INFINITY ? 0.f : -m_used;
+      uint8_t *pb = ps + buf * PBUF;
       float l4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
@@ -755,7 +818,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
         u.y = pack_bf16(p[2], p[3]);
         u.z = pack_bf16(p[4], p[5]);
         u.w = pack_bf16(p[6], p[7]);
-        *reinterpret_cast<uint4 *>(ps + row * 128 + (((c) ^ (row & 7)) << 4)) = u;
+        *reinterpret_cast<uint4 *>(pb + row * 128 + (((c) ^ (row & 7)) << 4)) = u;
       }
       l += (l4[0] + l4[1]) + (l4[2] + l4[3]);
       if (!blk && tile * 64 + 64 > n_keys) {
@@ -770,17 +833,13 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
       fence_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.p_ready);
+      if (lane == 0) mbar_arrive(&sm.p_ready[buf]);
     }
     if (!ok && lane == 0) set_status(status, DFLOW_ERR_DEVICE_TIMEOUT);
     // ---- this split's unnormalised O row, max and sum
     float o[128];
     if (ok && T > 0) {
-      int pv_ok = 1;
-      if (lane == 0) pv_ok = mbar_wait(&sm.pv_done, (uint32_t)((T - 1) & 1)) ? 1 : 0;
-      pv_ok = __shfl_sync(0xffffffffu, pv_ok, 0);
-      if (pv_ok) {
-        mbar_wait(&sm.pv_done, (uint32_t)((T - 1) & 1));
+      if (wait_all(&sm.pv_done[(T - 1) & 1], (uint32_t)(((T - 1) >> 1) & 1))) {
         tc_fence_after();
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld32(t_o + lane_off + c * 32, o + c * 32);
@@ -794,6 +853,8 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
     } else {
 #pragma unroll
       for (int j = 0; j < 128; ++j) o[j] = 0.f;
+      m_used = -INFINITY;
+      l = 0.f;
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");  // (B) every softmax warp has drained TMEM
     // the ring is reused for O once every copy and MMA has finished: wait for (A)
@@ -809,51 +870,75 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
   }
   if (warp < 2) __syncthreads();  // (A) for the producer and MMA warps
 
-  // ---- merge the splits of this cluster: CTA `split` finishes rows [r_lo, r_hi)
+  // ---- merge the splits of this cluster: CTA `split` finishes a slice of the valid rows
   __syncthreads();
   cluster_sync();
-  const int r_lo = split * T5_RPR;
-  if (threadIdx.x < T5_RPR) {
-    const int rr = r_lo + threadIdx.x;
-    float ms[T5_SPLITS], ls[T5_SPLITS], M = -INFINITY;
+  const int n_valid = min(QR - row0, T5_ROWS);
+  const int rpc = (n_valid + T5_SPLITS - 1) / T5_SPLITS;
+  const int r_lo = split * rpc, nr = max(min(r_lo + rpc, n_valid) - r_lo, 0);
+  const int units = nr * (HD / 4);
+  // one round trip of remote loads: thread t < 8 nr takes (row t / 8, split t % 8)'s
+  // max and sum; every thread takes the 8 split partials of up to two
+  // (row, 4-dim chunk) units
+  float mv = -INFINITY, lv = 0.f;
+  if (threadIdx.x < nr * T5_SPLITS) {
+    const int rr = r_lo + threadIdx.x / T5_SPLITS, sp = threadIdx.x % T5_SPLITS;
+    mv = ld_dsmem_f32(mapa(smem_u32(sm.m + rr), (uint32_t)sp));
+    lv = ld_dsmem_f32(mapa(smem_u32(sm.l + rr), (uint32_t)sp));
+  }
+  float4 x[2][T5_SPLITS];
+  auto load_units = [&](int u0) {
 #pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp) {
-      ms[sp] = ld_dsmem_f32(mapa(smem_u32(sm.m + rr), (uint32_t)sp));
-      ls[sp] = ld_dsmem_f32(mapa(smem_u32(sm.l + rr), (uint32_t)sp));
+    for (int h = 0; h < 2; ++h) {
+      const int u = u0 + h * THREADS;
+      if (u < units) {
+        const int rr = r_lo + u / (HD / 4), c4 = u % (HD / 4);
+        const int off = rr * HD + ((c4 ^ (rr & 7)) << 2);
+#pragma unroll
+        for (int sp = 0; sp < T5_SPLITS; ++sp) x[h][sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + off), (uint32_t)sp));
+      }
     }
+  };
+  load_units(threadIdx.x);
+  // merge weight of (row, split): 2^(m - M) / sum_s 2^(m_s - M) l_s over the 8
+  // lanes of the row (the Q tile is free now and holds them)
+  float *wsm = reinterpret_cast<float *>(qs);  // [rpc][T5_SPLITS]
+  {
+    float M = mv;
 #pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp) M = fmaxf(M, ms[sp]);
-    float L = 0.f;
+    for (int o = 1; o < T5_SPLITS; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    const float c = mv == -INFINITY ? 0.f : exp2f(mv - M);
+    float L = c * lv;
 #pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp) L += (ms[sp] == -INFINITY) ? 0.f : exp2f(ms[sp] - M) * ls[sp];
-#pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp)
-      sm.coef[threadIdx.x * T5_SPLITS + sp] = (ms[sp] == -INFINITY || L <= 0.f) ? 0.f : exp2f(ms[sp] - M) / L;
+    for (int o = 1; o < T5_SPLITS; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (threadIdx.x < nr * T5_SPLITS) wsm[threadIdx.x] = L > 0.f ? c / L : 0.f;
   }
   __syncthreads();
   bf16 *out = static_cast<bf16 *>(a.out);
-  for (int e = threadIdx.x; e < T5_RPR * (HD / 4); e += THREADS) {
-    const int rr = r_lo + e / (HD / 4), d4 = (e % (HD / 4)) * 4, q_r = row0 + rr;
-    if (q_r >= QR) continue;
-    float4 x[T5_SPLITS];
-    const int off = rr * HD + (((d4 >> 2) ^ (rr & 7)) << 2);
+  for (int u0 = threadIdx.x; u0 < units; u0 += 2 * THREADS) {
+    if (u0 != (int)threadIdx.x) load_units(u0);  // units past the first two per thread (a full 128-row group)
 #pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp) x[sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + off), (uint32_t)sp));
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int h = 0; h < 2; ++h) {
+      const int u = u0 + h * THREADS;
+      if (u >= units) continue;
+      const int rl = u / (HD / 4), d4 = (u % (HD / 4)) * 4, q_r = row0 + r_lo + rl;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int sp = 0; sp < T5_SPLITS; ++sp) {
-      const float c = sm.coef[(rr - r_lo) * T5_SPLITS + sp];
-      acc.x += c * x[sp].x;
-      acc.y += c * x[sp].y;
-      acc.z += c * x[sp].z;
-      acc.w += c * x[sp].w;
+      for (int sp = 0; sp < T5_SPLITS; ++sp) {
+        const float c = wsm[rl * T5_SPLITS + sp];
+        acc.x += c * x[h][sp].x;
+        acc.y += c * x[h][sp].y;
+        acc.z += c * x[h][sp].z;
+        acc.w += c * x[h][sp].w;
+      }
+      const int i = q_r / G, head = kvh * G + q_r % G;
+      bf16 *dst = out + ((size_t)(b * R + i) * D.hq + head) * HD + d4;
+      *reinterpret_cast<__nv_bfloat162 *>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
+      *reinterpret_cast<__nv_bfloat162 *>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
     }
-    const int i = q_r / G, head = kvh * G + q_r % G;
-    bf16 *dst = out + ((size_t)(b * R + i) * D.hq + head) * HD + d4;
-    *reinterpret_cast<__nv_bfloat162 *>(dst) = __floats2bfloat162_rn(acc.x, acc.y);
-    *reinterpret_cast<__nv_bfloat162 *>(dst + 2) = __floats2bfloat162_rn(acc.z, acc.w);
   }
   cluster_sync();  // peers may still read this CTA's shared memory until here
+  if (threadIdx.x == 0) dep_signal(a.dep);  // every global write of this CTA is done
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(T5_TMEM_COLS) : "memory");
@@ -861,9 +946,9 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, Dims D, AttnArgs a, int *statu
 }
 
 template <bool BLOCK>
-cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
-                      cudaStream_t s) {
-  const size_t smem = 1024 + 2 * T5_ROWS * 128 + T5_STAGES * 2 * (64 * 128 * 2) + T5_ROWS * 128 + sizeof(T5Smem);
+cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs a, int *status, cudaStream_t s,
+                      DepChain *chain) {
+  const size_t smem = 1024 + 2 * T5_ROWS * 128 + T5_STAGES * 2 * (64 * 128 * 2) + 2 * T5_ROWS * 128 + sizeof(T5Smem);
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(k_attn_t5<BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -872,6 +957,10 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, const Att
   }
   const int G = D.hq / D.hkv;
   const int qgroups = (D.R * G + T5_ROWS - 1) / T5_ROWS;
+  // one group of query rows: they arrive as two 3D boxes (64 dims x G heads x R rows)
+  CUtensorMap tq{};
+  const int q_tma = (qgroups == 1 && tensor_map_3d(&tq, a.q, D.hd, D.hq, batch * D.R, G, D.R)) ? 1 : 0;
+  a.dep = chain ? chain->take((unsigned)(D.hkv * batch * T5_SPLITS * qgroups)) : Dep{};
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(D.hkv, batch, T5_SPLITS * qgroups);
   cfg.blockDim = dim3(THREADS);
@@ -886,7 +975,7 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, const Att
   at[1].val.clusterDim.z = T5_SPLITS;
   cfg.attrs = at;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK>, tm, D, a, status);
+  return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK>, tm, tq, D, a, q_tma, status);
 }
 
 }  // namespace
@@ -895,7 +984,8 @@ bool attention_tc_supported(const Dims &D) {
   return D.page_size == 64 && (D.hd == 64 || D.hd == 128);
 }
 
-cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *status, cudaStream_t s) {
+cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *status, cudaStream_t s,
+                         DepChain *chain) {
   AttnArgs a = a_in;
   a.n_splits = MAX_SPLITS;  // one cluster of MAX_SPLITS key splits per (kv head, sequence, query group)
   CUtensorMap tm;
@@ -903,7 +993,9 @@ cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *st
   if (!tensor_map(&tm, a.pool, rows, D.hd, D.hd, 64)) return cudaErrorInvalidValue;
   const bool block = !a.causal;
   if (D.hd == 128 && getenv("DFLOW_MMA_SYNC_ATTENTION") == nullptr)
-    return block ? launch_t5<true>(tm, D, batch, a, status, s) : launch_t5<false>(tm, D, batch, a, status, s);
+    return block ? launch_t5<true>(tm, D, batch, a, status, s, chain)
+                 : launch_t5<false>(tm, D, batch, a, status, s, chain);
+  if (chain) chain->brk();
   if (D.hd == 128) return block ? launch<128, true>(tm, D, batch, a, status, s) : launch<128, false>(tm, D, batch, a, status, s);
   return block ? launch<64, true>(tm, D, batch, a, status, s) : launch<64, false>(tm, D, batch, a, status, s);
 }

@@ -74,6 +74,45 @@ inline cudaError_t klaunch(Kern kernel, dim3 grid, dim3 block, size_t smem, cuda
   return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+// Completion counters between consecutive launches of the tensor-core kernels
+// (GEMM, attention).  Every CTA of a launch adds 1 to the launch's counter
+// (release) once all its global writes are done; a launch that directly
+// follows such a launch acquires that counter until it reaches the previous
+// launch's CTA count, instead of waiting for the previous grid to be torn down.
+// Counters are cumulative across launches that share a slot.
+struct Dep {
+  const unsigned int *wait;  // previous launch's counter, or null: griddepcontrol.wait
+  unsigned int wait_n;       // its value once every CTA of the previous launch is done
+  unsigned int *signal;      // this launch's counter, or null
+};
+
+// Host side of the counters of one handle (its calls are issued in order on one
+// stream).  A launch that counts takes the next slot; it waits on the previous
+// slot only when the launch right before it counted too (brk() after any other
+// launch).  Slots are reused round robin, their expected values accumulating.
+constexpr int kDepSlots = 64;
+struct DepChain {
+  unsigned int *dev = nullptr;          // [kDepSlots] counters in device memory
+  unsigned int shadow[kDepSlots] = {};  // value of each counter once every launch so far is done
+  int last = -1;                        // slot of the previous launch when it counted, else -1
+  int next = 0;
+  bool dirty = true;                    // counters and shadow disagree: zero both before use
+  Dep take(unsigned int n_ctas) {
+    Dep d{};
+    if (dev == nullptr) return d;
+    if (last >= 0) {
+      d.wait = dev + last;
+      d.wait_n = shadow[last];
+    }
+    last = next;
+    next = (next + 1) % kDepSlots;
+    shadow[last] += n_ctas;
+    d.signal = dev + last;
+    return d;
+  }
+  void brk() { last = -1; }
+};
+
 // ---------------------------------------------------------------------------
 // GEMM: out[m][n] = sum_k X[m][k] * W[n][k] with a fused epilogue
 // ---------------------------------------------------------------------------
@@ -163,10 +202,14 @@ struct AttnArgs {
   int n_splits;
   float *part;            // [rows][hq][n_splits][hd + 2]
   void *out;              // [rows][hq * hd]
+  Dep dep;                // completion counters (tcgen05 kernel only)
 };
-cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s);
+// chain: completion counters of the caller's launch sequence, or null
+cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s,
+                      DepChain *chain = nullptr);
 // tensor-core path for bf16 caches with 64-token pages (attn_tc.cu)
 bool attention_tc_supported(const Dims &D);
-cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s);
+cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s,
+                         DepChain *chain = nullptr);
 
 }  // namespace dflow

@@ -54,6 +54,7 @@ struct Params {
   uint32_t idesc;
   EpArgs ep;
   int *status;
+  Dep dep;
 };
 
 struct Smem {
@@ -270,7 +271,7 @@ template <int EP>
 __global__ void __launch_bounds__(THREADS, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const Params p) {
   // the next kernel may launch once every CTA of this one runs; inputs produced by
-  // the previous kernel are read only after pdl_wait() (weights are prefetched before it)
+  // the previous launch are read only after dep_wait() (weights are prefetched before it)
   pdl_trigger();
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
@@ -326,7 +327,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         tma_load_2d(ring + (size_t)u * stage_bytes, &tmW, (kr0 + u % nk) * BK, (q + (u / nk) * p.Q) * BM, &sm.full[u], pw);
       }
       n_issued = pre;
-      pdl_wait();
+      dep_wait(p.dep, p.status);
+      if (p.dep.wait) fence_proxy_async_global();
       for (int u = 0; u < pre; ++u)
         tma_load_2d(ring + (size_t)u * stage_bytes + A_BYTES, &tmX, (kr0 + u % nk) * BK, 0, &sm.full[u], px);
       stage = pre % p.stages;
@@ -400,7 +402,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
-    pdl_wait();
+    if (leader) dep_wait(p.dep, p.status);
+    epi_bar();  // the other epilogue threads read the previous launch's outputs after the leader's wait
     if (p.ep.in_ss) {
       // the input rows' RMSNorm, folded into a per-column scale of the product
       for (int c = r; c < p.M; c += BM) {
@@ -545,6 +548,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   __syncwarp();  // lanes that skipped a single-thread role wait for it here
   tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 0) dep_signal(p.dep);  // every global write of this CTA is done
   if (p.P > 1) cluster_sync();  // no CTA leaves while a peer may still read its shared memory
   if (warp == 1) {
     tc_fence_after();
@@ -668,13 +672,15 @@ Choice choose(int T, int kb, int npad, int sm_count, bool use_cache) {
 }
 
 template <int EP>
-cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_count, cudaStream_t s, bool use_cache) {
+cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_count, cudaStream_t s, bool use_cache,
+                DepChain *chain) {
   const Choice c = choose<EP>(p.T, p.kb, p.npad, sm_count, use_cache);
   if (c.P == 0) return cudaErrorInvalidValue;
   p.P = c.P;
   p.Q = c.Q;
   p.stages = c.stages;
   p.red_ld = c.red_ld;
+  p.dep = chain ? chain->take((unsigned)(c.P * c.Q)) : Dep{};
   return launch_ep<EP>(mw, mx, p, c.smem, s);
 }
 
@@ -741,6 +747,17 @@ bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, i
   return true;
 }
 
+bool tensor_map_3d(CUtensorMap *out, const void *ptr, int d0, int d1, int d2, int b1, int b2) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = encode_fn();
+  if (!enc || b1 < 1 || b2 < 1 || b1 > 256 || b2 > 256) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)d0, (cuuint64_t)d1, (cuuint64_t)d2};
+  cuuint64_t strides[2] = {(cuuint64_t)d0 * 2, (cuuint64_t)d0 * d1 * 2};
+  cuuint32_t box[3] = {(cuuint32_t)BK, (cuuint32_t)b1, (cuuint32_t)b2};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max, int max_tiles) {
   (void)base;
@@ -762,7 +779,7 @@ cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s) {
 }
 
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
-                    const EpArgs &ep_in, int *status, cudaStream_t s, bool use_caches) {
+                    const EpArgs &ep_in, int *status, cudaStream_t s, bool use_caches, DepChain *chain) {
   CUtensorMap mw;
   if (!tensor_map(&mw, W, N, K, K, BM, use_caches)) return cudaErrorInvalidValue;
   for (int m0 = 0; m0 < M; m0 += MAX_NPAD) {
@@ -797,12 +814,12 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
       return cudaErrorInvalidValue;
     cudaError_t e;
     switch (ep.mode) {
-      case EP_STORE_F32: e = run<EP_STORE_F32>(mw, mx, p, w.sm_count, s, use_caches); break;
-      case EP_RESID: e = run<EP_RESID>(mw, mx, p, w.sm_count, s, use_caches); break;
-      case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s, use_caches); break;
-      case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s, use_caches); break;
-      case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s, use_caches); break;
-      case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s, use_caches); break;
+      case EP_STORE_F32: e = run<EP_STORE_F32>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      case EP_RESID: e = run<EP_RESID>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      case EP_SWIGLU: e = run<EP_SWIGLU>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;

@@ -9,6 +9,9 @@ namespace dflow {
 // 2D tensor map of a bf16 row-major [rows][ld] matrix, box 64 columns x box_rows
 // rows, 128-byte swizzle (cached by arguments).
 bool tensor_map(CUtensorMap *out, const void *ptr, int rows, int cols, int ld, int box_rows, bool use_cache = true);
+// 3D tensor map of a bf16 [d2][d1][d0] array (d0 contiguous), box 64 x b1 x b2,
+// 128-byte swizzle (not cached)
+bool tensor_map_3d(CUtensorMap *out, const void *ptr, int d0, int d1, int d2, int b1, int b2);
 
 // Scratch of the tensor-core GEMM inside the handle's workspace.
 struct TcWorkspace {
@@ -27,7 +30,9 @@ bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep);
 cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s);
 // use_caches = false: tensor maps are encoded on the stack and the launch plan
 // is recomputed, so the call touches no host heap
+// chain: completion counters of the caller's launch sequence, or null (grid waits)
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M,
-                    int ldx, const EpArgs &ep, int *status, cudaStream_t s, bool use_caches = true);
+                    int ldx, const EpArgs &ep, int *status, cudaStream_t s, bool use_caches = true,
+                    DepChain *chain = nullptr);
 
 }  // namespace dflow

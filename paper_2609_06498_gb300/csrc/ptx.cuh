@@ -3,6 +3,8 @@
 #include <cuda.h>
 #include <stdint.h>
 
+#include "dflow_internal.cuh"
+
 namespace dflow {
 namespace ptx {
 
@@ -60,6 +62,16 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int x, int y, int z, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 // K-major operand, 128-byte swizzle: 8-row groups 1024 bytes apart
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
@@ -148,6 +160,34 @@ __device__ __forceinline__ float ld_dsmem_f32(uint32_t caddr) {
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+
+// ---- completion counters between consecutive launches (see Dep)
+// Waits until the previous launch's counter shows every one of its CTAs done
+// (acquire), or, with no counter, for the previous grid (griddepcontrol.wait).
+// Bounded: on expiry the status records DFLOW_ERR_DEVICE_TIMEOUT and the
+// caller carries on (its results are then void).
+__device__ __forceinline__ void dep_wait(const Dep &d, int *status) {
+  if (d.wait == nullptr) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    return;
+  }
+  const unsigned long long t0 = gtime();
+  for (int i = 0;; ++i) {
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(d.wait) : "memory");
+    if ((int)(v - d.wait_n) >= 0) return;
+    if ((i & 15) == 15 && gtime() - t0 > WAIT_NS) {
+      atomicCAS(status, 0, (int)DFLOW_ERR_DEVICE_TIMEOUT);
+      return;
+    }
+  }
+}
+// this CTA's completion (one thread, after a barrier over every thread that wrote)
+__device__ __forceinline__ void dep_signal(const Dep &d) {
+  if (d.signal != nullptr) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(d.signal) : "memory");
+}
+// global data made visible to this thread by an acquire, to its later TMA reads
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
 }  // namespace ptx
 }  // namespace dflow

@@ -137,3 +137,25 @@ def test_full_depth_8b_round_invariants():
         assert bd[0] == gk[a] and bd[1] == (bk[a + 1] if a < B else -1)
         assert np.isfinite(to_np(feats)).all()
     assert eng.read_status(st) == 0
+
+
+def test_batch16_long_context_rounds_stay_clean():
+    """Forty rounds of the batch-16, 8K-context shape (2 + 1 layers, full widths):
+    no bounded device wait may expire, and every sequence grows by exactly its
+    forced acceptance + 1 per round (Eq. 3).  Exercises every pipeline barrier of
+    the attention and GEMM kernels over several hundred launches."""
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = reduced(synth.QWEN3_8B_KV)
+    rounds = 40
+    max_ctx = cfg.replace(new_tokens=rounds * cfg.rows).max_ctx()
+    eng = Engine(cfg, random_weights(cfg, seed=0), max_batch=cfg.batch, max_ctx=max_ctx)
+    st = eng.new_state(cfg.batch, page_seed=0)
+    eng.prefill(st, synth.prompts(cfg))
+    assert eng.read_status(st) == 0
+    n0 = to_np(st.seq_len).astype(np.int64)
+    sched = synth.forced_schedule(cfg, rounds)
+    for r in range(rounds):
+        eng.round(st, torch.as_tensor(sched[r]).cuda())
+    assert eng.read_status(st) == 0
+    assert np.array_equal(to_np(st.seq_len).astype(np.int64), n0 + (sched + 1).sum(axis=0))
