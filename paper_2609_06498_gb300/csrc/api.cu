@@ -665,6 +665,30 @@ EpArgs qkv_ep(const dflow_handle *h, const Dims &D, int nq, const float *qn, con
   return e;
 }
 
+// attention of one layer: q (h->q) against the layer's pool (and, drafter, the
+// block's own K/V) into h->ao
+cudaError_t layer_attention(const Call &k, const Dims &D, int batch, void *pool_layer, const dflow_state *st,
+                            int causal, int splits) {
+  dflow_handle *h = k.h;
+  const int rows = batch * D.R;
+  AttnArgs a{};
+  a.q = h->q;
+  a.pool = pool_layer;
+  a.page_table = st->page_table;
+  a.bk = causal ? nullptr : h->bk;
+  a.bv = causal ? nullptr : h->bv;
+  a.pos = h->pos;
+  a.seq_len = st->seq_len;
+  a.kvlen = h->kvlen;
+  a.causal = causal;
+  a.n_splits = splits;
+  a.part = h->apart;
+  a.out = h->ao;
+  ProfScope ps(h, k.s, DFLOW_PROF_ATTN, 0.0, 4.0 * rows * D.hq * D.hd);
+  h->n_launch += 1;
+  return attention(h->dtype, D, batch, a, k.status_w, k.s, &h->dep);
+}
+
 // One Qwen3 decoder layer over `rows` rows held in h->x (fp32 residual).
 //   causal = 1: target layer; K/V written to the paged pool (rows with wr),
 //               attention over positions 0..pos.
@@ -693,24 +717,7 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
                          causal ? nullptr : h->bv)))
       return e;
   }
-  AttnArgs a{};
-  a.q = h->q;
-  a.pool = pool_layer;
-  a.page_table = st->page_table;
-  a.bk = causal ? nullptr : h->bk;
-  a.bv = causal ? nullptr : h->bv;
-  a.pos = h->pos;
-  a.seq_len = st->seq_len;
-  a.kvlen = h->kvlen;
-  a.causal = causal;
-  a.n_splits = splits;
-  a.part = h->apart;
-  a.out = h->ao;
-  {
-    ProfScope ps(h, k.s, DFLOW_PROF_ATTN, 0.0, 4.0 * rows * D.hq * D.hd);
-    h->n_launch += 2;
-    if ((e = attention(h->dtype, D, batch, a, k.status_w, k.s, &h->dep))) return e;
-  }
+  if ((e = layer_attention(k, D, batch, pool_layer, st, causal, splits))) return e;
   if (h->fused) {
     if ((e = gemm(k, L.w_o, D.d, qd, h->ao, rows, qd, resid_norm(h, L.mlp_norm, nullptr)))) return e;
     if ((e = gemm(k, L.w_gate_up, 2 * D.inter, D.d, h->xn, rows, D.d, in_norm(ep_t(EP_SWIGLU, h->mlp, D.inter), h))))
@@ -761,6 +768,54 @@ void *stash_slot(const dflow_handle *h, int l) {
   return nullptr;
 }
 
+// The decoder layers [0, nL) of one stack (target: causal, K/V to its pool and
+// the Eq. 1 stash; drafter: block K/V) over the rows in h->x, layer by layer.
+// With DFLOW_SEQ_GEMMS set (fused tensor-core path, few rows) the first QKV
+// projection runs alone, then each layer is its attention plus one persistent
+// launch of its O, gate/up and down projections and the next layer's QKV.
+template <typename T>
+cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_layer_weights *Ls, int nL,
+                          T *pool_base, const dflow_state *st, int causal, int splits, const float *final_gain) {
+  dflow_handle *h = k.h;
+  const int rows = batch * D.R, qkv_dim = (D.hq + 2 * D.hkv) * D.hd, qd = D.hq * D.hd;
+  auto pool = [&](int l) { return pool_base + (size_t)l * pool_layer_elems(D); };
+  auto next_gain = [&](int l) { return l + 1 < nL ? Ls[l + 1].attn_norm : final_gain; };
+  auto stash = [&](int l) { return causal ? stash_slot<T>(h, l) : nullptr; };
+  // (opt-in while the per-tile split-K epilogue, not the weight stream, bounds it)
+  const bool seq = h->fused && h->dep.dev != nullptr && seq_supported(rows) && getenv("DFLOW_SEQ_GEMMS") != nullptr;
+  cudaError_t e;
+  if (!seq) {
+    for (int l = 0; l < nL; ++l)
+      if ((e = layer_forward<T>(k, D, batch, Ls[l], pool(l), st, causal, splits, next_gain(l), stash(l)))) return e;
+    return cudaSuccess;
+  }
+  auto qkv_args = [&](int l) {
+    return in_norm(qkv_ep(h, D, D.hq, Ls[l].q_norm, Ls[l].k_norm, h->pos, h->wr, causal ? (void *)pool(l) : nullptr,
+                          st->page_table, !causal),
+                   h);
+  };
+  if ((e = gemm(k, Ls[0].w_qkv, qkv_dim, D.d, h->xn, rows, D.d, qkv_args(0)))) return e;
+  for (int l = 0; l < nL; ++l) {
+    if ((e = layer_attention(k, D, batch, pool(l), st, causal, splits))) return e;
+    const dflow_layer_weights &L = Ls[l];
+    SeqSpec sp[4];
+    int n = 0;
+    sp[n++] = SeqSpec{L.w_o, D.d, qd, h->ao, qd, resid_norm(h, L.mlp_norm, nullptr)};
+    sp[n++] = SeqSpec{L.w_gate_up, 2 * D.inter, D.d, h->xn, D.d, in_norm(ep_t(EP_SWIGLU, h->mlp, D.inter), h)};
+    sp[n++] = SeqSpec{L.w_down, D.d, D.inter, h->mlp, D.inter, resid_norm(h, next_gain(l), stash(l))};
+    if (l + 1 < nL) sp[n++] = SeqSpec{Ls[l + 1].w_qkv, qkv_dim, D.d, h->xn, D.d, qkv_args(l + 1)};
+    double bytes = 0.0, flops = 0.0;
+    for (int j = 0; j < n; ++j) {
+      bytes += (double)h->esz * sp[j].N * sp[j].K + (double)h->esz * rows * sp[j].K + ep_out_bytes(sp[j].ep, rows, sp[j].N, h->esz);
+      flops += 2.0 * rows * sp[j].N * sp[j].K;
+    }
+    ProfScope ps(h, k.s, DFLOW_PROF_GEMM, bytes, flops);
+    ++h->n_launch;
+    if ((e = gemm_seq(h->tcw, n, sp, rows, k.status_w, k.s, &h->dep))) return e;
+  }
+  return cudaSuccess;
+}
+
 // target forward over h->x (embeddings) at h->pos; writes K/V, g, Eq. 1 features
 template <typename T>
 cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_state *st, int *g,
@@ -769,11 +824,9 @@ cudaError_t target_forward(const Call &k, const Dims &D, int batch, const dflow_
   const int rows = batch * D.R;
   const int L = h->cfg.n_layers;
   cudaError_t e;
-  for (int l = 0; l < L; ++l) {
-    T *pool_l = static_cast<T *>(st->kv) + (size_t)l * pool_layer_elems(D);
-    const float *next_gain = l + 1 < L ? h->tl[l + 1].attn_norm : h->w.final_norm;
-    if ((e = layer_forward<T>(k, D, batch, h->tl[l], pool_l, st, 1, splits, next_gain, stash_slot<T>(h, l)))) return e;
-  }
+  if ((e = stack_forward<T>(k, D, batch, h->tl.data(), L, static_cast<T *>(st->kv), st, 1, splits,
+                            h->w.final_norm)))
+    return e;
   if ((e = lm_head_argmax<T>(k, D, rows, h->w.final_norm, g, logits))) return e;
   // Eq. 1: H_T = RMSNorm(W_c [H^l1; ...; H^lm])
   if ((e = gemm(k, h->w.w_c, D.d, D.n_feat * D.d, h->stash, rows, D.n_feat * D.d, ep_f32(h->gf32, h->gld)))) return e;
@@ -832,12 +885,8 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
                                           k.status));
   CK(cudaGetLastError());
   const int splits = pick_splits(h, batch, rows);
-  const int Ld = h->cfg.draft_layers;
-  for (int l = 0; l < Ld; ++l) {
-    T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
-    const float *next_gain = l + 1 < Ld ? h->dl[l + 1].attn_norm : h->w.draft_final_norm;
-    CK(layer_forward<T>(k, D, batch, h->dl[l], pool_l, st, 0, splits, next_gain, nullptr));
-  }
+  CK(stack_forward<T>(k, D, batch, h->dl.data(), h->cfg.draft_layers, static_cast<T *>(st->draft_kv), st, 0, splits,
+                      h->w.draft_final_norm));
   CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
   KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
                                                    D.R, blk, k.status));

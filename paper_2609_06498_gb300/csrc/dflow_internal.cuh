@@ -110,6 +110,15 @@ struct DepChain {
     d.signal = dev + last;
     return d;
   }
+  // a counter for completions inside one launch (the chain's last slot is unchanged)
+  unsigned int *alloc(unsigned int n, unsigned int *target) {
+    if (dev == nullptr) return nullptr;
+    const int s = next;
+    next = (next + 1) % kDepSlots;
+    shadow[s] += n;
+    *target = shadow[s];
+    return dev + s;
+  }
   void brk() { last = -1; }
 };
 

@@ -97,9 +97,10 @@ __device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const f
   epi_bar();
 }
 
-// prefetch of the inputs epilogue_chunk(t, c0, nc) will need
-template <int EP>
-__device__ __forceinline__ void epilogue_prefetch(const Params &p, const Smem &sm, int t, int r, int c0, int nc,
+// prefetch of the inputs epilogue_chunk(t, c0, nc) will need (PT: any parameter
+// block with the GEMM's N, M and ep)
+template <int EP, typename PT>
+__device__ __forceinline__ void epilogue_prefetch(const PT &p, const Smem &sm, int t, int r, int c0, int nc,
                                                   EpPre &pre) {
   const EpArgs &ep = p.ep;
   const int n = t * BM + r, ncol = min(c0 + nc, p.M) - c0;
@@ -120,8 +121,8 @@ __device__ __forceinline__ void epilogue_prefetch(const Params &p, const Smem &s
 }
 
 // epilogue on token columns c0 .. c0+nc-1 (nc <= 16) of tile t; v[j] = D[row r][c0+j]
-template <int EP>
-__device__ __forceinline__ void epilogue_chunk(const Params &p, Smem &sm, int t, int r, int sub, int lane, int c0,
+template <int EP, typename PT>
+__device__ __forceinline__ void epilogue_chunk(const PT &p, Smem &sm, int t, int r, int sub, int lane, int c0,
                                                int nc, float *v, const EpPre &pre) {
   const int n = t * BM + r;
   const EpArgs &ep = p.ep;
@@ -556,6 +557,430 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   }
 }
 
+// ===========================================================================
+// Persistent sequence of weight-streaming GEMMs: one launch per layer segment
+// (O, gate/up, down projections and the next layer's QKV projection).  One
+// cluster of SEQ_P CTAs owns 128-row tiles q, q + Q, ... of every GEMM and
+// splits their K range as k_gemm_tc does.  The producer streams weight
+// k-blocks without a break across the GEMM boundaries; a unit's activation
+// k-block is issued once every tile of the previous GEMM is finished (one
+// completion counter per GEMM, one release add per CTA and tile), so the next
+// GEMM's weights fill the ring while the epilogue warps finish the current
+// GEMM.  Every CTA of the grid is resident at once (the grid is sized by the
+// cluster occupancy), which the cross-CTA waits rely on.
+// ===========================================================================
+constexpr int SEQ_MAX = 4;  // GEMMs per launch
+constexpr int SEQ_P = 4;    // cluster size = split-K ways
+
+struct SeqGemm {
+  int N, K, M, T, kb, mode;
+  uint32_t idesc;
+  EpArgs ep;
+  unsigned int *done;   // completion counter: +1 per CTA and finished tile
+  unsigned int done_n;  // its value once every tile of this GEMM is finished
+};
+struct SeqMaps {
+  CUtensorMap w[SEQ_MAX], x[SEQ_MAX];  // weights [N][K], activations [M][K]
+};
+struct SeqParams {
+  int n, M, npad, Q, stages, tmem_cols, red_ld;
+  int *status;
+  Dep dep;  // the previous launch: inputs of the first GEMM
+  SeqGemm g[SEQ_MAX];
+};
+
+__device__ __forceinline__ bool counter_reached(const unsigned int *c, unsigned int n) {
+  unsigned int v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(c) : "memory");
+  return (int)(v - n) >= 0;
+}
+// bounded wait on a completion counter (acquire); false on expiry
+__device__ __forceinline__ bool counter_wait(const unsigned int *c, unsigned int n) {
+  const unsigned long long t0 = gtime();
+  for (int i = 0;; ++i) {
+    if (counter_reached(c, n)) return true;
+    if ((i & 15) == 15 && gtime() - t0 > WAIT_NS) return false;
+  }
+}
+__device__ __forceinline__ void counter_add(unsigned int *c) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(c) : "memory");
+}
+
+// the tensor maps of GEMM j, addressed with constant offsets into the parameter block
+__device__ __forceinline__ const CUtensorMap *seq_wmap(const SeqMaps &m, int j) {
+  switch (j) {
+    case 0: return &m.w[0];
+    case 1: return &m.w[1];
+    case 2: return &m.w[2];
+    default: return &m.w[3];
+  }
+}
+__device__ __forceinline__ const CUtensorMap *seq_xmap(const SeqMaps &m, int j) {
+  switch (j) {
+    case 0: return &m.x[0];
+    case 1: return &m.x[1];
+    case 2: return &m.x[2];
+    default: return &m.x[3];
+  }
+}
+
+// this CTA's tile count and k-block range of every GEMM, read once from the
+// parameter block with constant indices and kept in registers (the unit loops
+// index them through sel4, never with a runtime array index)
+struct SeqTab {
+  int n, nt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX];
+};
+__device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
+  return j == 0 ? a[0] : j == 1 ? a[1] : j == 2 ? a[2] : a[3];
+}
+__device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int q, int rank) {
+  SeqTab t;
+  t.n = p.n;
+#pragma unroll
+  for (int j = 0; j < SEQ_MAX; ++j) {
+    const bool on = j < p.n;
+    t.nt[j] = on && p.g[j].T > q ? (p.g[j].T - 1 - q) / p.Q + 1 : 0;
+    t.k0[j] = on ? rank * p.g[j].kb / SEQ_P : 0;
+    t.k1[j] = on ? (rank + 1) * p.g[j].kb / SEQ_P : 0;
+  }
+  return t;
+}
+
+// cursor over this CTA's units (GEMM j, tile index ti, k-block k); j == n: past the end
+struct SeqCur {
+  int j, ti, k;
+};
+__device__ __forceinline__ void seq_skip_empty(const SeqTab &tb, SeqCur &c) {
+  while (c.j < tb.n && sel4(tb.nt, c.j) == 0) ++c.j;
+  c.ti = 0;
+  if (c.j < tb.n) c.k = sel4(tb.k0, c.j);
+}
+__device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
+  if (++c.k < sel4(tb.k1, c.j)) return;
+  c.k = sel4(tb.k0, c.j);
+  if (++c.ti < sel4(tb.nt, c.j)) return;
+  ++c.j;
+  seq_skip_empty(tb, c);
+}
+
+// the split-K epilogue of one tile (the k_gemm_tc path with P = SEQ_P), then
+// this CTA's completion mark for the tile; false when a bounded wait expired
+template <int EP>
+__device__ __forceinline__ bool seq_tile_epilogue(const SeqGemm &g, Smem &sm, float *red, int red_ld, int npad,
+                                               uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rank,
+                                               bool leader, int s0, int s1) {
+  const int buf = i & 1;
+  EpPre pre;
+  epilogue_prefetch<EP>(g, sm, t, r, s0, min(16, s1 - s0), pre);
+  if (leader) {
+    int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
+    if (ok && i > 0) ok = mbar_wait_cluster(&sm.freeb, (i - 1) & 1) ? 1 : 0;
+    sm.flag = ok;
+  }
+  __syncwarp();
+  epi_bar();
+  if (!sm.flag) return false;
+  tc_fence_after();
+  const uint32_t acc_addr = lane_addr + buf * npad;
+  float v[16];
+  // park this CTA's fp32 partial in its shared memory (row r, contiguous columns)
+  float *mine = red + (size_t)r * red_ld;
+  for (int c0 = 0; c0 < npad && c0 < g.M; c0 += 16) {
+    tmem_ld16(acc_addr + c0, v);
+#pragma unroll
+    for (int j = 0; j < 16; j += 4)
+      *reinterpret_cast<float4 *>(mine + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+  }
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(&sm.acce[buf]);
+  epi_bar();
+  if (leader) {
+#pragma unroll
+    for (int pr = 0; pr < SEQ_P; ++pr)
+      if (pr != rank) mbar_arrive_remote(&sm.ready, (uint32_t)pr);
+    sm.flag = mbar_wait_cluster(&sm.ready, i & 1) ? 1 : 0;
+  }
+  __syncwarp();
+  epi_bar();
+  const bool ok = sm.flag != 0;
+  bool released = false;
+  if (ok) {
+    const uint32_t my_row = smem_u32(mine);
+    for (int c0 = s0; c0 < s1; c0 += 16) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = 0.f;
+      // the SEQ_P partials in fixed rank order (deterministic), all loads in flight together
+      float4 x[SEQ_P][4];
+#pragma unroll
+      for (int gi = 0; gi < SEQ_P; ++gi) {
+        const uint32_t base = mapa(my_row, (uint32_t)gi);
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4)
+          x[gi][q4] = c0 + 4 * q4 < s1 ? ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int gi = 0; gi < SEQ_P; ++gi) {
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          v[4 * q4] += x[gi][q4].x;
+          v[4 * q4 + 1] += x[gi][q4].y;
+          v[4 * q4 + 2] += x[gi][q4].z;
+          v[4 * q4 + 3] += x[gi][q4].w;
+        }
+      }
+      if (c0 + 16 >= s1) {
+        // the last remote reads of this tile are done: the peers may overwrite their partials
+        epi_bar();
+        if (leader)
+#pragma unroll
+          for (int pr = 0; pr < SEQ_P; ++pr)
+            if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+        released = true;
+      }
+      if (c0 > s0) epilogue_prefetch<EP>(g, sm, t, r, c0, min(16, s1 - c0), pre);
+      epilogue_chunk<EP>(g, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
+    }
+  }
+  if (!released) {
+    epi_bar();  // this CTA has finished reading every peer's partial
+    if (leader)
+#pragma unroll
+      for (int pr = 0; pr < SEQ_P; ++pr)
+        if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
+  }
+  epi_bar();  // every epilogue thread's stores of the tile are done (and sm.flag may be rewritten)
+  if (ok && leader) counter_add(g.done);
+  return ok;
+}
+
+constexpr int SEQ_THREADS = THREADS + 32;  // warp 6: the activation producer
+
+__global__ void __launch_bounds__(SEQ_THREADS, 1)
+k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqParams p) {
+  // the next launch may start once every CTA of this one runs; it waits on the
+  // last GEMM's completion counter
+  pdl_trigger();
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
+  const int stage_bytes = A_BYTES + p.npad * BK * 2;
+  float *red = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [BM][red_ld]
+  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(red) + (size_t)BM * p.red_ld * 4);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int rank = (int)cluster_rank();
+  const int q = blockIdx.x / SEQ_P;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&sm.full[s], 2);  // one arrival (with its byte count) from each producer
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.accf[b], 1);
+      mbar_init(&sm.acce[b], 4);
+    }
+    mbar_init(&sm.ready, SEQ_P - 1);
+    mbar_init(&sm.freeb, SEQ_P - 1);
+    mbar_init(&sm.drain, 1);
+    sm.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
+                 "r"(p.tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // peers' barriers are initialised before anyone signals them
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem;
+
+  if (warp == 0 || warp == 6) {
+    // ---------------- TMA producers: warp 0 streams every unit's weight k-block
+    // (nothing to wait for but a free stage, so the next GEMM's weights fill the
+    // ring ahead of time); warp 6 its activation k-block, once the GEMM's inputs
+    // are complete.  Each arrives on the stage's full barrier with its own bytes.
+    if (lane == 0) {
+      const bool wp = warp == 0;
+      const SeqTab tb = seq_tab(p, q, rank);
+      const uint64_t pol = wp ? policy_evict_first() : policy_evict_last();
+      const uint32_t bytes = wp ? (uint32_t)A_BYTES : (uint32_t)(stage_bytes - A_BYTES);
+      if (wp)
+        for (int j = 0; j < tb.n; ++j) prefetch_tensormap(seq_wmap(maps, j));
+      int stage = 0, u = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (int j = 0; j < tb.n && ok; ++j) {
+        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j);
+        if (nt == 0) continue;
+        const CUtensorMap *map = wp ? seq_wmap(maps, j) : seq_xmap(maps, j);
+        if (!wp) {
+          // GEMM j reads what GEMM j - 1 (or the previous launch) wrote
+          if (j == 0) {
+            dep_wait(p.dep, p.status);
+          } else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n)) {
+            ok = false;
+            break;
+          }
+          if (j > 0 || p.dep.wait) fence_proxy_async_global();
+          prefetch_tensormap(map);
+        }
+        for (int ti = 0; ti < nt && ok; ++ti) {
+          const int row = wp ? (q + ti * p.Q) * BM : 0;
+          for (int k = k0; k < k1; ++k, ++u) {
+            if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
+              ok = false;
+              break;
+            }
+            mbar_expect_tx(&sm.full[stage], bytes);
+            tma_load_2d(ring + (size_t)stage * stage_bytes + (wp ? 0 : A_BYTES), map, k * BK, row, &sm.full[stage], pol);
+            if (++stage == p.stages) {
+              stage = 0;
+              ph ^= 1;
+            }
+          }
+        }
+      }
+      if (!ok) {
+        set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+        atomicExch(&sm.abort, 1);
+      }
+      // this producer's copies have landed before the CTA may exit: each of the
+      // last `stages` units' full barrier completes once both producers' bytes are in
+      if (wp && ok) {
+        for (int v = u > p.stages ? u - p.stages : 0; v < u; ++v)
+          if (!mbar_wait(&sm.full[v % p.stages], (uint32_t)((v / p.stages) & 1)))
+            set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+      } else if (!ok) {
+        // an aborted launch: stages may lack the other producer's copy, so give
+        // this producer's copies a bounded time to land
+        const unsigned long long t0 = gtime();
+        while (gtime() - t0 < 200000ull) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      int i = 0;
+      const SeqTab tb = seq_tab(p, q, rank);
+      const uint32_t idesc = p.g[0].idesc;  // one row count, so one instruction descriptor for all GEMMs
+      for (int j = 0; j < tb.n && ok; ++j) {
+        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j);
+        for (int ti = 0; ti < nt && ok; ++ti, ++i) {
+          const int buf = i & 1;
+          if (!mbar_wait(&sm.acce[buf], ((i >> 1) & 1) ^ 1)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t d = tmem + buf * p.npad;
+          for (int k = k0; k < k1; ++k) {
+            if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t a = smem_u32(ring + (size_t)stage * stage_bytes);
+            const uint64_t ad = smem_desc(a), bd = smem_desc(a + A_BYTES);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (k > k0 || kk > 0) ? 1u : 0u);
+            mma_commit(&sm.empty[stage]);
+            if (++stage == p.stages) {
+              stage = 0;
+              ph ^= 1;
+            }
+          }
+          if (!ok) break;
+          mma_commit(&sm.accf[buf]);
+        }
+      }
+      if (!ok) {
+        set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+        atomicExch(&sm.abort, 1);
+      }
+      mma_commit(&sm.drain);
+      if (!mbar_wait(&sm.drain, 0)) set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+    }
+  } else {
+    // ---------------- epilogue warps 2..5 ----------------
+    const int sub = warp & 3;
+    const int r = sub * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
+    const bool leader = threadIdx.x == 64;
+    const int w4 = ((p.M + 4 * SEQ_P - 1) / (4 * SEQ_P)) * 4;
+    const int s0 = min(rank * w4, p.M), s1 = min((rank + 1) * w4, p.M);
+    const SeqTab tb = seq_tab(p, q, rank);
+    bool ok = true;
+    int i = 0;
+    for (int j = 0; j < p.n && ok; ++j) {
+      const SeqGemm &g = p.g[j];
+      // every input of this GEMM's epilogue (norm partials, residual, positions) is
+      // in place once the previous GEMM, or the previous launch, is finished
+      if (leader) {
+        if (j == 0)
+          dep_wait(p.dep, p.status);
+        else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n))
+          set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+      }
+      epi_bar();
+      if (g.ep.in_ss) {
+        // the input rows' RMSNorm, folded into a per-column scale of the product
+        for (int c = r; c < p.M; c += BM) {
+          float acc = 0.f;
+          for (int e = 0; e < g.ep.in_ss_n; ++e) acc += __ldcg(g.ep.in_ss + (size_t)e * g.ep.ld_ss + c);
+          sm.col_scale[c] = rsqrtf(acc * g.ep.in_inv_d + g.ep.in_eps);
+        }
+        epi_bar();
+      }
+      if (g.mode == EP_QKV) {
+        const QkvOut &o = g.ep.qkv;
+        for (int c = r; c < p.M; c += BM) {
+          const int grow = o.row0 + c, pp = o.pos[grow];
+          long long base = -1;
+          if (o.bk == nullptr && o.wr[grow]) {
+            const int page = o.page_table[(size_t)(grow / o.R) * o.pages_per_seq + pp / o.page_size];
+            base = ((long long)page * 2 * o.hkv * o.page_size + pp % o.page_size) * BM;
+          }
+          sm.qkv_pos[c] = pp;
+          sm.qkv_base[c] = base;
+        }
+        epi_bar();
+      }
+      const int nt = sel4(tb.nt, j);
+      for (int ti = 0; ti < nt && ok; ++ti, ++i) {
+        const int t = q + ti * p.Q;
+        switch (g.mode) {
+          case EP_RESID:
+            ok = seq_tile_epilogue<EP_RESID>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            break;
+          case EP_SWIGLU:
+            ok = seq_tile_epilogue<EP_SWIGLU>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            break;
+          case EP_QKV:
+            ok = seq_tile_epilogue<EP_QKV>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            break;
+          default:
+            ok = seq_tile_epilogue<EP_STORE_F32>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            break;
+        }
+      }
+    }
+    if (!ok && leader) {
+      set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+      atomicExch(&sm.abort, 1);
+    }
+  }
+
+  __syncwarp();  // lanes that skipped a single-thread role wait for it here
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while a peer may still read its shared memory
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
+  }
+}
+
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
@@ -682,6 +1107,45 @@ cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_c
   p.red_ld = c.red_ld;
   p.dep = chain ? chain->take((unsigned)(c.P * c.Q)) : Dep{};
   return launch_ep<EP>(mw, mx, p, c.smem, s);
+}
+
+size_t seq_smem(int npad, int *stages_out, int *red_ld_out) {
+  const int stage_bytes = A_BYTES + npad * BK * 2;
+  const int red_ld = npad + 4;
+  const size_t red_bytes = (size_t)BM * red_ld * 4;
+  int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
+  if (stages > 16) stages = 16;
+  *stages_out = stages;
+  *red_ld_out = red_ld;
+  return 1024 + (size_t)stages * stage_bytes + red_bytes + sizeof(Smem);
+}
+
+// clusters of SEQ_P persistent CTAs that are resident at once
+int seq_clusters(size_t smem) {
+  static std::mutex mu;
+  static std::map<size_t, int> cache;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(smem);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (cudaFuncSetAttribute(k_gemm_seq, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048) ==
+      cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(SEQ_P);
+    cfg.blockDim = dim3(SEQ_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = SEQ_P;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k_gemm_seq, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();
+  cache.emplace(smem, n);
+  return n;
 }
 
 }  // namespace
@@ -825,6 +1289,70 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+bool seq_supported(int M) {
+  return M >= 1 && (M + 15) / 16 * 16 <= MAX_SPLIT_NPAD && encode_fn() != nullptr;
+}
+
+cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
+                     DepChain *chain) {
+  (void)w;
+  if (n < 1 || n > SEQ_MAX || !chain || !chain->dev || !seq_supported(M)) return cudaErrorInvalidValue;
+  SeqParams p{};
+  SeqMaps maps{};
+  p.n = n;
+  p.M = M;
+  p.npad = (M + 15) / 16 * 16;
+  p.status = status;
+  int cols = 32;
+  while (cols < 2 * p.npad) cols <<= 1;
+  p.tmem_cols = cols;
+  const size_t smem = seq_smem(p.npad, &p.stages, &p.red_ld);
+  p.Q = seq_clusters(smem);
+  if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
+  const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+  for (int j = 0; j < n; ++j) {
+    const SeqSpec &q = sp[j];
+    const int mode = q.ep.mode;
+    if (q.K % BK || q.K / BK < SEQ_P || q.N < 1 || q.ldx % 8 ||
+        (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV))
+      return cudaErrorInvalidValue;
+    SeqGemm &g = p.g[j];
+    g.N = q.N;
+    g.K = q.K;
+    g.M = M;
+    g.T = (q.N + BM - 1) / BM;
+    g.kb = q.K / BK;
+    g.mode = mode;
+    g.idesc = idesc;
+    g.ep = q.ep;
+    g.ep.qkv.row0 = 0;
+    if (!tensor_map(&maps.w[j], q.W, q.N, q.K, q.K, BM) || !tensor_map(&maps.x[j], q.X, M, q.K, q.ldx, p.npad))
+      return cudaErrorInvalidValue;
+  }
+  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc((unsigned)(SEQ_P * p.g[j].T), &p.g[j].done_n);
+  const Dep d = chain->take((unsigned)(SEQ_P * p.g[n - 1].T));
+  p.g[n - 1].done = d.signal;
+  p.g[n - 1].done_n = chain->shadow[chain->last];
+  p.dep = d;
+  p.dep.signal = nullptr;
+
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.Q * SEQ_P);
+  cfg.blockDim = dim3(SEQ_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = SEQ_P;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, k_gemm_seq, maps, p);
 }
 
 }  // namespace dflow

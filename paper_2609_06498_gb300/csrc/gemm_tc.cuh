@@ -35,4 +35,21 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
                     int ldx, const EpArgs &ep, int *status, cudaStream_t s, bool use_caches = true,
                     DepChain *chain = nullptr);
 
+// One GEMM of a persistent sequence (out[m][n] = X[m][:] . W[n][:] with a
+// fused epilogue; modes EP_STORE_F32, EP_RESID, EP_SWIGLU, EP_QKV).
+struct SeqSpec {
+  const void *W;
+  int N, K;
+  const void *X;
+  int ldx;
+  EpArgs ep;
+};
+// True when up to 4 GEMMs over M rows can run as one persistent launch.
+bool seq_supported(int M);
+// The GEMMs of `sp` in order, in one launch: GEMM j's activations are read once
+// every tile of GEMM j - 1 is finished; the first waits for the previous launch
+// in `chain` (required), the next launch waits for the last GEMM.
+cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
+                     DepChain *chain);
+
 }  // namespace dflow

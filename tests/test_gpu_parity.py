@@ -195,6 +195,16 @@ def test_round_parity(setup):
     assert exact_rounds >= cfg.batch * 4
 
 
+def test_round_parity_persistent_gemms(setup, monkeypatch):
+    """The same rounds with each layer's O, gate/up, down and next-QKV projections
+    in one persistent launch (the bf16 path with 128-dim heads, few rows)."""
+    cfg = setup[0]
+    if cfg.dtype != "bf16" or cfg.head_dim != 128:
+        pytest.skip("persistent GEMM sequence: bf16 with 128-dim heads")
+    monkeypatch.setenv("DFLOW_SEQ_GEMMS", "1")
+    test_round_parity(setup)
+
+
 def test_generate_matches_oracle_tiny():
     """fp32: the whole generation (prefill + natural-acceptance rounds) equals the
     oracle's, which the oracle tests pin to plain greedy decoding."""
