@@ -50,7 +50,7 @@ constexpr int THREADS = 192;
 constexpr int SMEM_BUDGET = 224 * 1024;
 
 struct Params {
-  int N, K, M, npad, T, kb, P, Q, stages, tmem_cols, red_ld;
+  int N, K, M, npad, T, kb, P, Q, stages, tmem_cols, rx_bytes;
   uint32_t idesc;
   EpArgs ep;
   int *status;
@@ -58,7 +58,10 @@ struct Params {
 };
 
 struct Smem {
-  uint64_t full[16], empty[16], accf[2], acce[2], ready, freeb, drain;
+  // recv: this CTA's slice of the split-K partials has arrived (armed by the CTA
+  // itself, completed by its peers' bytes); rfree: every owner has consumed
+  // this CTA's previous pushes (one arrival per peer)
+  uint64_t full[16], empty[16], accf[2], acce[2], recv, rfree, drain;
   uint32_t tmem;
   int flag;
   int abort;
@@ -268,6 +271,100 @@ __device__ __forceinline__ void epilogue_chunk(const PT &p, Smem &sm, int t, int
   }
 }
 
+// 16 bytes into a peer CTA's shared memory, counted on the peer's barrier
+__device__ __forceinline__ void st_async_f4(uint32_t caddr, const float4 &v, uint32_t cbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(caddr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(cbar)
+               : "memory");
+}
+// split-K: token columns [s0, s1) of rank `rank` out of P (4-column groups)
+__device__ __forceinline__ int splitk_w4(int M, int P) { return ((M + 4 * P - 1) / (4 * P)) * 4; }
+// bytes the owner of [s0, s1) receives per tile: a float4 per row and column group from each peer
+__device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
+  return s1 > s0 ? (uint32_t)((P - 1) * BM * ((s1 - s0 + 3) / 4) * 16) : 0u;
+}
+
+// One tile of a P-way split-K GEMM (P > 1).  Every CTA of the cluster holds a
+// partial of the whole [128 x M] tile; rank r finishes token columns [s0, s1).
+// Each thread pushes its row's partial, 4-column group by group, into the
+// receive area of the group's owner (st.async, counted on the owner's recv
+// barrier; its own groups locally), frees the TMEM buffer, then waits for its
+// own recv barrier alone, sums the P partials in rank order (deterministic) and
+// runs the fused epilogue.  It re-arms recv for the next tile before telling
+// the senders (rfree) that they may push again.  False when a wait expired.
+template <int EP, typename PT>
+__device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P, int npad, int M,
+                                            uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rank,
+                                            bool leader) {
+  const int w4 = splitk_w4(M, P);
+  const int s0 = min(rank * w4, M), s1 = min((rank + 1) * w4, M);
+  const int buf = i & 1;
+  EpPre pre;
+  epilogue_prefetch<EP>(g, sm, t, r, s0, min(16, s1 - s0), pre);
+  if (leader) {
+    int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
+    if (ok && i > 0) ok = mbar_wait_cluster(&sm.rfree, (i - 1) & 1) ? 1 : 0;
+    sm.flag = ok;
+  }
+  __syncwarp();
+  epi_bar();
+  if (!sm.flag) return false;
+  tc_fence_after();
+  const uint32_t acc_addr = lane_addr + buf * npad;
+  const uint32_t rx_s = smem_u32(rx), recv_s = smem_u32(&sm.recv);
+  float v[16];
+  for (int c0 = 0; c0 < npad && c0 < M; c0 += 16) {
+    tmem_ld16(acc_addr + c0, v);
+#pragma unroll
+    for (int q4 = 0; q4 < 4; ++q4) {
+      const int col = c0 + 4 * q4;
+      if (col >= M) break;
+      const int owner = col / w4;
+      const int e = (rank * BM + r) * w4 + (col - owner * w4);  // the sender's slot in the owner's area
+      const float4 x = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+      if (owner == rank)
+        *reinterpret_cast<float4 *>(rx + e) = x;
+      else
+        st_async_f4(mapa(rx_s + (uint32_t)e * 4, (uint32_t)owner), x, mapa(recv_s, (uint32_t)owner));
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(&sm.acce[buf]);
+  if (leader) sm.flag = mbar_wait(&sm.recv, i & 1) ? 1 : 0;
+  __syncwarp();
+  epi_bar();
+  const bool ok = sm.flag != 0;
+  if (ok) {
+    for (int c0 = s0; c0 < s1; c0 += 16) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) v[j] = 0.f;
+      for (int sp = 0; sp < P; ++sp) {
+        const float *src = rx + (sp * BM + r) * w4 + (c0 - s0);
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          if (c0 + 4 * q4 >= s1) break;
+          const float4 y = *reinterpret_cast<const float4 *>(src + 4 * q4);
+          v[4 * q4] += y.x;
+          v[4 * q4 + 1] += y.y;
+          v[4 * q4 + 2] += y.z;
+          v[4 * q4 + 3] += y.w;
+        }
+      }
+      if (c0 > s0) epilogue_prefetch<EP>(g, sm, t, r, c0, min(16, s1 - c0), pre);
+      epilogue_chunk<EP>(g, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
+    }
+  }
+  epi_bar();  // every thread has read the receive area (and sm.flag may be rewritten)
+  if (leader) {
+    mbar_expect_tx(&sm.recv, splitk_recv_bytes(P, s0, s1));  // armed before any sender may push again
+#pragma unroll 1
+    for (int pr = 0; pr < P; ++pr)
+      if (pr != rank) mbar_arrive_remote(&sm.rfree, (uint32_t)pr);
+  }
+  return ok;
+}
+
 template <int EP>
 __global__ void __launch_bounds__(THREADS, 1)
 k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX, const Params p) {
@@ -277,8 +374,8 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
-  float *red = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [BM][red_ld] (P > 1)
-  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(red) + (p.P > 1 ? (size_t)BM * p.red_ld * 4 : 0));
+  float *rx = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [P][BM][w4] split-K receive area
+  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(rx) + p.rx_bytes);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int rank = p.P > 1 ? (int)cluster_rank() : 0;
   const int q = blockIdx.x / p.P;
@@ -293,11 +390,16 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       mbar_init(&sm.accf[b], 1);
       mbar_init(&sm.acce[b], 4);
     }
-    mbar_init(&sm.ready, p.P > 1 ? p.P - 1 : 1);
-    mbar_init(&sm.freeb, p.P > 1 ? p.P - 1 : 1);
+    mbar_init(&sm.recv, 1);
+    mbar_init(&sm.rfree, p.P > 1 ? p.P - 1 : 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (p.P > 1) {
+      // armed for the first tile before the cluster barrier below lets any peer push
+      const int w4 = splitk_w4(p.M, p.P);
+      mbar_expect_tx(&sm.recv, splitk_recv_bytes(p.P, min(rank * w4, p.M), min((rank + 1) * w4, p.M)));
+    }
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
@@ -429,33 +531,25 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
       }
       epi_bar();
     }
-    // token columns this CTA finishes after the split-K reduction (multiple of 4)
-    const int w4 = ((p.M + 4 * p.P - 1) / (4 * p.P)) * 4;
-    const int s0 = min(rank * w4, p.M), s1 = min((rank + 1) * w4, p.M);
-    const int c_first = p.P == 1 ? 0 : s0;
     int i = 0;
     for (int t = q; t < p.T; t += p.Q, ++i) {
       const int buf = i & 1;
-      EpPre pre;
-      epilogue_prefetch<EP>(p, sm, t, r, c_first, p.P == 1 ? 16 : min(16, s1 - s0), pre);
-      if (leader) {
-        int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
-        if (ok && p.P > 1 && i > 0) ok = mbar_wait_cluster(&sm.freeb, (i - 1) & 1) ? 1 : 0;
-        sm.flag = ok;
-      }
-      __syncwarp();
-      epi_bar();
-      if (!sm.flag) {
-        if (leader) {
-          set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
-          atomicExch(&sm.abort, 1);
-        }
-        break;
-      }
-      tc_fence_after();
-      const uint32_t acc_addr = lane_addr + buf * p.npad;
-      float v[16];
       if (p.P == 1) {
+        EpPre pre;
+        epilogue_prefetch<EP>(p, sm, t, r, 0, 16, pre);
+        if (leader) sm.flag = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
+        __syncwarp();
+        epi_bar();
+        if (!sm.flag) {
+          if (leader) {
+            set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+            atomicExch(&sm.abort, 1);
+          }
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc_addr = lane_addr + buf * p.npad;
+        float v[16];
         for (int c0 = 0; c0 < p.npad && c0 < p.M; c0 += 16) {
           if (c0 > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
           tmem_ld16(acc_addr + c0, v);
@@ -465,76 +559,7 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
       } else {
-        // park this CTA's fp32 partial in its shared memory (row r, contiguous columns)
-        float *mine = red + (size_t)r * p.red_ld;
-        for (int c0 = 0; c0 < p.npad && c0 < p.M; c0 += 16) {
-          tmem_ld16(acc_addr + c0, v);
-#pragma unroll
-          for (int j = 0; j < 16; j += 4)
-            *reinterpret_cast<float4 *>(mine + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.acce[buf]);
-        epi_bar();
-        if (leader) {
-          for (int pr = 0; pr < p.P; ++pr)
-            if (pr != rank) mbar_arrive_remote(&sm.ready, (uint32_t)pr);
-          sm.flag = mbar_wait_cluster(&sm.ready, i & 1) ? 1 : 0;
-        }
-        __syncwarp();
-        epi_bar();
-        const bool ok = sm.flag != 0;
-        bool released = false;
-        if (ok) {
-          const uint32_t my_row = smem_u32(mine);
-          for (int c0 = s0; c0 < s1; c0 += 16) {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) v[j] = 0.f;
-            // peers in groups of four, fixed rank order (deterministic); a group's remote
-            // loads are all in flight together
-            for (int g0 = 0; g0 < p.P; g0 += 4) {
-              float4 x[4][4];
-#pragma unroll
-              for (int gi = 0; gi < 4; ++gi) {
-                const uint32_t base = mapa(my_row, (uint32_t)min(g0 + gi, p.P - 1));
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4)
-                  x[gi][q4] = (g0 + gi < p.P && c0 + 4 * q4 < s1) ? ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4)
-                                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
-              }
-#pragma unroll
-              for (int gi = 0; gi < 4; ++gi) {
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                  v[4 * q4] += x[gi][q4].x;
-                  v[4 * q4 + 1] += x[gi][q4].y;
-                  v[4 * q4 + 2] += x[gi][q4].z;
-                  v[4 * q4 + 3] += x[gi][q4].w;
-                }
-              }
-            }
-            if (c0 + 16 >= s1) {
-              // the last remote reads of this tile are done: the peers may overwrite their
-              // partials.  Signalled before the epilogue's global stores, which a release
-              // arrive after them would have to wait for.
-              epi_bar();
-              if (leader)
-                for (int pr = 0; pr < p.P; ++pr)
-                  if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
-              released = true;
-            }
-            if (c0 > s0) epilogue_prefetch<EP>(p, sm, t, r, c0, min(16, s1 - c0), pre);
-            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
-          }
-        }
-        if (!released) {
-          epi_bar();  // this CTA has finished reading every peer's partial
-          if (leader)
-            for (int pr = 0; pr < p.P; ++pr)
-              if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
-        }
-        if (!ok) {
+        if (!splitk_tile<EP>(p, sm, rx, p.P, p.npad, p.M, lane_addr, i, t, r, sub, lane, rank, leader)) {
           if (leader) {
             set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
             atomicExch(&sm.abort, 1);
@@ -583,7 +608,7 @@ struct SeqMaps {
   CUtensorMap w[SEQ_MAX], x[SEQ_MAX];  // weights [N][K], activations [M][K]
 };
 struct SeqParams {
-  int n, M, npad, Q, stages, tmem_cols, red_ld;
+  int n, M, npad, Q, stages, tmem_cols, rx_bytes;
   int *status;
   Dep dep;  // the previous launch: inputs of the first GEMM
   SeqGemm g[SEQ_MAX];
@@ -663,93 +688,13 @@ __device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
   seq_skip_empty(tb, c);
 }
 
-// the split-K epilogue of one tile (the k_gemm_tc path with P = SEQ_P), then
-// this CTA's completion mark for the tile; false when a bounded wait expired
+// one tile of GEMM g (split-K over the cluster), then this CTA's completion mark
+// for the tile; false when a bounded wait expired
 template <int EP>
-__device__ __forceinline__ bool seq_tile_epilogue(const SeqGemm &g, Smem &sm, float *red, int red_ld, int npad,
-                                               uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rank,
-                                               bool leader, int s0, int s1) {
-  const int buf = i & 1;
-  EpPre pre;
-  epilogue_prefetch<EP>(g, sm, t, r, s0, min(16, s1 - s0), pre);
-  if (leader) {
-    int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
-    if (ok && i > 0) ok = mbar_wait_cluster(&sm.freeb, (i - 1) & 1) ? 1 : 0;
-    sm.flag = ok;
-  }
-  __syncwarp();
-  epi_bar();
-  if (!sm.flag) return false;
-  tc_fence_after();
-  const uint32_t acc_addr = lane_addr + buf * npad;
-  float v[16];
-  // park this CTA's fp32 partial in its shared memory (row r, contiguous columns)
-  float *mine = red + (size_t)r * red_ld;
-  for (int c0 = 0; c0 < npad && c0 < g.M; c0 += 16) {
-    tmem_ld16(acc_addr + c0, v);
-#pragma unroll
-    for (int j = 0; j < 16; j += 4)
-      *reinterpret_cast<float4 *>(mine + c0 + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
-  }
-  tc_fence_before();
-  __syncwarp();
-  if (lane == 0) mbar_arrive(&sm.acce[buf]);
-  epi_bar();
-  if (leader) {
-#pragma unroll
-    for (int pr = 0; pr < SEQ_P; ++pr)
-      if (pr != rank) mbar_arrive_remote(&sm.ready, (uint32_t)pr);
-    sm.flag = mbar_wait_cluster(&sm.ready, i & 1) ? 1 : 0;
-  }
-  __syncwarp();
-  epi_bar();
-  const bool ok = sm.flag != 0;
-  bool released = false;
-  if (ok) {
-    const uint32_t my_row = smem_u32(mine);
-    for (int c0 = s0; c0 < s1; c0 += 16) {
-#pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = 0.f;
-      // the SEQ_P partials in fixed rank order (deterministic), all loads in flight together
-      float4 x[SEQ_P][4];
-#pragma unroll
-      for (int gi = 0; gi < SEQ_P; ++gi) {
-        const uint32_t base = mapa(my_row, (uint32_t)gi);
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4)
-          x[gi][q4] = c0 + 4 * q4 < s1 ? ld_dsmem_f4(base + (uint32_t)(c0 + 4 * q4) * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int gi = 0; gi < SEQ_P; ++gi) {
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          v[4 * q4] += x[gi][q4].x;
-          v[4 * q4 + 1] += x[gi][q4].y;
-          v[4 * q4 + 2] += x[gi][q4].z;
-          v[4 * q4 + 3] += x[gi][q4].w;
-        }
-      }
-      if (c0 + 16 >= s1) {
-        // the last remote reads of this tile are done: the peers may overwrite their partials
-        epi_bar();
-        if (leader)
-#pragma unroll
-          for (int pr = 0; pr < SEQ_P; ++pr)
-            if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
-        released = true;
-      }
-      if (c0 > s0) epilogue_prefetch<EP>(g, sm, t, r, c0, min(16, s1 - c0), pre);
-      epilogue_chunk<EP>(g, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
-    }
-  }
-  if (!released) {
-    epi_bar();  // this CTA has finished reading every peer's partial
-    if (leader)
-#pragma unroll
-      for (int pr = 0; pr < SEQ_P; ++pr)
-        if (pr != rank) mbar_arrive_remote(&sm.freeb, (uint32_t)pr);
-  }
-  epi_bar();  // every epilogue thread's stores of the tile are done (and sm.flag may be rewritten)
+__device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, int npad, uint32_t lane_addr, int i,
+                                         int t, int r, int sub, int lane, int rank, bool leader) {
+  const bool ok = splitk_tile<EP>(g, sm, rx, SEQ_P, npad, g.M, lane_addr, i, t, r, sub, lane, rank, leader);
+  epi_bar();  // every epilogue thread's stores of the tile are done
   if (ok && leader) counter_add(g.done);
   return ok;
 }
@@ -764,8 +709,8 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
-  float *red = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [BM][red_ld]
-  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(red) + (size_t)BM * p.red_ld * 4);
+  float *rx = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [SEQ_P][BM][w4] split-K receive area
+  Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(rx) + p.rx_bytes);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int rank = (int)cluster_rank();
   const int q = blockIdx.x / SEQ_P;
@@ -779,11 +724,13 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       mbar_init(&sm.accf[b], 1);
       mbar_init(&sm.acce[b], 4);
     }
-    mbar_init(&sm.ready, SEQ_P - 1);
-    mbar_init(&sm.freeb, SEQ_P - 1);
+    mbar_init(&sm.recv, 1);
+    mbar_init(&sm.rfree, SEQ_P - 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    const int w4 = splitk_w4(p.M, SEQ_P);
+    mbar_expect_tx(&sm.recv, splitk_recv_bytes(SEQ_P, min(rank * w4, p.M), min((rank + 1) * w4, p.M)));
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
@@ -907,8 +854,6 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
-    const int w4 = ((p.M + 4 * SEQ_P - 1) / (4 * SEQ_P)) * 4;
-    const int s0 = min(rank * w4, p.M), s1 = min((rank + 1) * w4, p.M);
     const SeqTab tb = seq_tab(p, q, rank);
     bool ok = true;
     int i = 0;
@@ -951,16 +896,16 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         const int t = q + ti * p.Q;
         switch (g.mode) {
           case EP_RESID:
-            ok = seq_tile_epilogue<EP_RESID>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            ok = seq_tile<EP_RESID>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
             break;
           case EP_SWIGLU:
-            ok = seq_tile_epilogue<EP_SWIGLU>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            ok = seq_tile<EP_SWIGLU>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
             break;
           case EP_QKV:
-            ok = seq_tile_epilogue<EP_QKV>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            ok = seq_tile<EP_QKV>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
             break;
           default:
-            ok = seq_tile_epilogue<EP_STORE_F32>(g, sm, red, p.red_ld, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, s0, s1);
+            ok = seq_tile<EP_STORE_F32>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
             break;
         }
       }
@@ -1049,7 +994,7 @@ int max_clusters(int P, size_t smem, bool use_cache) {
 }
 
 struct Choice {
-  int P = 0, Q = 0, stages = 0, red_ld = 0;
+  int P = 0, Q = 0, stages = 0, rx_bytes = 0;
   size_t smem = 0;
 };
 
@@ -1069,8 +1014,8 @@ Choice choose(int T, int kb, int npad, int sm_count, bool use_cache) {
   long best_cost = -1;
   for (int P : {1, 2, 3, 4, 6, 8}) {
     if (P > kb || (P > 1 && npad > MAX_SPLIT_NPAD)) continue;
-    const int red_ld = npad + 4;
-    const size_t red_bytes = P > 1 ? (size_t)BM * red_ld * 4 : 0;
+    // split-K receive area: P slots of [BM][w4] floats (w4 bounded with npad >= M)
+    const size_t red_bytes = P > 1 ? (size_t)P * BM * (((npad + 4 * P - 1) / (4 * P)) * 4) * 4 : 0;
     int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
     if (stages > 16) stages = 16;
     if (stages < 3) continue;
@@ -1085,7 +1030,7 @@ Choice choose(int T, int kb, int npad, int sm_count, bool use_cache) {
       best.P = P;
       best.Q = Q;
       best.stages = stages;
-      best.red_ld = red_ld;
+      best.rx_bytes = (int)red_bytes;
       best.smem = smem;
     }
   }
@@ -1104,19 +1049,18 @@ cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_c
   p.P = c.P;
   p.Q = c.Q;
   p.stages = c.stages;
-  p.red_ld = c.red_ld;
+  p.rx_bytes = c.rx_bytes;
   p.dep = chain ? chain->take((unsigned)(c.P * c.Q)) : Dep{};
   return launch_ep<EP>(mw, mx, p, c.smem, s);
 }
 
-size_t seq_smem(int npad, int *stages_out, int *red_ld_out) {
+size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
   const int stage_bytes = A_BYTES + npad * BK * 2;
-  const int red_ld = npad + 4;
-  const size_t red_bytes = (size_t)BM * red_ld * 4;
+  const size_t red_bytes = (size_t)SEQ_P * BM * (((npad + 4 * SEQ_P - 1) / (4 * SEQ_P)) * 4) * 4;
   int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
   if (stages > 16) stages = 16;
   *stages_out = stages;
-  *red_ld_out = red_ld;
+  *rx_bytes_out = (int)red_bytes;
   return 1024 + (size_t)stages * stage_bytes + red_bytes + sizeof(Smem);
 }
 
@@ -1308,7 +1252,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   int cols = 32;
   while (cols < 2 * p.npad) cols <<= 1;
   p.tmem_cols = cols;
-  const size_t smem = seq_smem(p.npad, &p.stages, &p.red_ld);
+  const size_t smem = seq_smem(p.npad, &p.stages, &p.rx_bytes);
   p.Q = seq_clusters(smem);
   if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
   const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
