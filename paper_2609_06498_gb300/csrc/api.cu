@@ -769,10 +769,11 @@ void *stash_slot(const dflow_handle *h, int l) {
 }
 
 // The decoder layers [0, nL) of one stack (target: causal, K/V to its pool and
-// the Eq. 1 stash; drafter: block K/V) over the rows in h->x, layer by layer.
-// With DFLOW_SEQ_GEMMS set (fused tensor-core path, few rows) the first QKV
-// projection runs alone, then each layer is its attention plus one persistent
-// launch of its O, gate/up and down projections and the next layer's QKV.
+// the Eq. 1 stash; drafter: block K/V) over the rows in h->x.  On the fused
+// tensor-core path with few rows the first QKV projection runs alone, then each
+// layer is its attention plus one persistent launch of its O, gate/up and down
+// projections and the next layer's QKV; otherwise (or with
+// DFLOW_SEPARATE_GEMMS set) layer by layer, one launch per projection.
 template <typename T>
 cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_layer_weights *Ls, int nL,
                           T *pool_base, const dflow_state *st, int causal, int splits, const float *final_gain) {
@@ -781,8 +782,8 @@ cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_l
   auto pool = [&](int l) { return pool_base + (size_t)l * pool_layer_elems(D); };
   auto next_gain = [&](int l) { return l + 1 < nL ? Ls[l + 1].attn_norm : final_gain; };
   auto stash = [&](int l) { return causal ? stash_slot<T>(h, l) : nullptr; };
-  // (opt-in while the per-tile split-K epilogue, not the weight stream, bounds it)
-  const bool seq = h->fused && h->dep.dev != nullptr && seq_supported(rows) && getenv("DFLOW_SEQ_GEMMS") != nullptr;
+  const bool seq =
+      h->fused && h->dep.dev != nullptr && seq_supported(rows) && getenv("DFLOW_SEPARATE_GEMMS") == nullptr;
   cudaError_t e;
   if (!seq) {
     for (int l = 0; l < nL; ++l)

@@ -335,6 +335,19 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
   __syncwarp();
   epi_bar();
   const bool ok = sm.flag != 0;
+  // re-arm recv for the next tile, then let the senders push again; done right
+  // after the last read of the receive area, before the epilogue's global
+  // stores (which a release arrive issued after them would wait for)
+  auto release = [&]() {
+    epi_bar();  // every thread has read the receive area
+    if (leader) {
+      mbar_expect_tx(&sm.recv, splitk_recv_bytes(P, s0, s1));
+#pragma unroll 1
+      for (int pr = 0; pr < P; ++pr)
+        if (pr != rank) mbar_arrive_remote_relaxed(&sm.rfree, (uint32_t)pr);
+    }
+  };
+  bool released = false;
   if (ok) {
     for (int c0 = s0; c0 < s1; c0 += 16) {
 #pragma unroll
@@ -351,17 +364,15 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
           v[4 * q4 + 3] += y.w;
         }
       }
+      if (c0 + 16 >= s1) {
+        release();
+        released = true;
+      }
       if (c0 > s0) epilogue_prefetch<EP>(g, sm, t, r, c0, min(16, s1 - c0), pre);
       epilogue_chunk<EP>(g, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
     }
   }
-  epi_bar();  // every thread has read the receive area (and sm.flag may be rewritten)
-  if (leader) {
-    mbar_expect_tx(&sm.recv, splitk_recv_bytes(P, s0, s1));  // armed before any sender may push again
-#pragma unroll 1
-    for (int pr = 0; pr < P; ++pr)
-      if (pr != rank) mbar_arrive_remote(&sm.rfree, (uint32_t)pr);
-  }
+  if (!released) release();
   return ok;
 }
 
@@ -601,7 +612,7 @@ struct SeqGemm {
   int N, K, M, T, kb, mode;
   uint32_t idesc;
   EpArgs ep;
-  unsigned int *done;   // completion counter: +1 per CTA and finished tile
+  unsigned int *done;   // completion counter: each CTA adds its tile count once its tiles are finished
   unsigned int done_n;  // its value once every tile of this GEMM is finished
 };
 struct SeqMaps {
@@ -627,8 +638,8 @@ __device__ __forceinline__ bool counter_wait(const unsigned int *c, unsigned int
     if ((i & 15) == 15 && gtime() - t0 > WAIT_NS) return false;
   }
 }
-__device__ __forceinline__ void counter_add(unsigned int *c) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(c) : "memory");
+__device__ __forceinline__ void counter_add(unsigned int *c, unsigned int n) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(c), "r"(n) : "memory");
 }
 
 // the tensor maps of GEMM j, addressed with constant offsets into the parameter block
@@ -688,14 +699,12 @@ __device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
   seq_skip_empty(tb, c);
 }
 
-// one tile of GEMM g (split-K over the cluster), then this CTA's completion mark
-// for the tile; false when a bounded wait expired
+// one tile of GEMM g (split-K over the cluster); false when a bounded wait expired
 template <int EP>
 __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, int npad, uint32_t lane_addr, int i,
                                          int t, int r, int sub, int lane, int rank, bool leader) {
   const bool ok = splitk_tile<EP>(g, sm, rx, SEQ_P, npad, g.M, lane_addr, i, t, r, sub, lane, rank, leader);
-  epi_bar();  // every epilogue thread's stores of the tile are done
-  if (ok && leader) counter_add(g.done);
+  epi_bar();  // sm.flag is rewritten at the top of the next tile
   return ok;
 }
 
@@ -909,6 +918,8 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
             break;
         }
       }
+      // this CTA's share of GEMM j is written (a barrier over the epilogue threads above)
+      if (ok && leader && nt > 0) counter_add(g.done, (unsigned int)nt);
     }
     if (!ok && leader) {
       set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);

@@ -195,13 +195,13 @@ def test_round_parity(setup):
     assert exact_rounds >= cfg.batch * 4
 
 
-def test_round_parity_persistent_gemms(setup, monkeypatch):
-    """The same rounds with each layer's O, gate/up, down and next-QKV projections
-    in one persistent launch (the bf16 path with 128-dim heads, few rows)."""
+def test_round_parity_separate_gemms(setup, monkeypatch):
+    """The same rounds with one launch per projection instead of the persistent
+    per-layer launch the bf16 path with 128-dim heads and few rows takes."""
     cfg = setup[0]
     if cfg.dtype != "bf16" or cfg.head_dim != 128:
-        pytest.skip("persistent GEMM sequence: bf16 with 128-dim heads")
-    monkeypatch.setenv("DFLOW_SEQ_GEMMS", "1")
+        pytest.skip("the persistent GEMM sequence is the bf16 path with 128-dim heads")
+    monkeypatch.setenv("DFLOW_SEPARATE_GEMMS", "1")
     test_round_parity(setup)
 
 
