@@ -284,20 +284,22 @@ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
   return s1 > s0 ? (uint32_t)((P - 1) * BM * ((s1 - s0 + 3) / 4) * 16) : 0u;
 }
 
-// One tile of a P-way split-K GEMM (P > 1).  Every CTA of the cluster holds a
-// partial of the whole [128 x M] tile; rank r finishes token columns [s0, s1).
+// One tile of a P-way split-K GEMM (P > 1) done by the P CTAs at cluster ranks
+// rbase .. rbase + P - 1 (this CTA is the rr-th).  Every one holds a partial of
+// the whole [128 x M] tile; the rr-th finishes token columns [s0, s1).
 // Each thread pushes its row's partial, 4-column group by group, into the
 // receive area of the group's owner (st.async, counted on the owner's recv
 // barrier; its own groups locally), frees the TMEM buffer, then waits for its
 // own recv barrier alone, sums the P partials in rank order (deterministic) and
-// runs the fused epilogue.  It re-arms recv for the next tile before telling
-// the senders (rfree) that they may push again.  False when a wait expired.
+// runs the fused epilogue.  It re-arms recv with next_bytes (what its next
+// split-K tile will receive) before telling the senders (rfree, rfree_n
+// arrivals each) that they may push again.  False when a wait expired.
 template <int EP, typename PT>
 __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P, int npad, int M,
-                                            uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rank,
-                                            bool leader) {
+                                            uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
+                                            int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n) {
   const int w4 = splitk_w4(M, P);
-  const int s0 = min(rank * w4, M), s1 = min((rank + 1) * w4, M);
+  const int s0 = min(rr * w4, M), s1 = min((rr + 1) * w4, M);
   const int buf = i & 1;
   EpPre pre;
   epilogue_prefetch<EP>(g, sm, t, r, s0, min(16, s1 - s0), pre);
@@ -320,12 +322,12 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
       const int col = c0 + 4 * q4;
       if (col >= M) break;
       const int owner = col / w4;
-      const int e = (rank * BM + r) * w4 + (col - owner * w4);  // the sender's slot in the owner's area
+      const int e = (rr * BM + r) * w4 + (col - owner * w4);  // the sender's slot in the owner's area
       const float4 x = make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
-      if (owner == rank)
+      if (owner == rr)
         *reinterpret_cast<float4 *>(rx + e) = x;
       else
-        st_async_f4(mapa(rx_s + (uint32_t)e * 4, (uint32_t)owner), x, mapa(recv_s, (uint32_t)owner));
+        st_async_f4(mapa(rx_s + (uint32_t)e * 4, (uint32_t)(rbase + owner)), x, mapa(recv_s, (uint32_t)(rbase + owner)));
     }
   }
   tc_fence_before();
@@ -341,10 +343,10 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
   auto release = [&]() {
     epi_bar();  // every thread has read the receive area
     if (leader) {
-      mbar_expect_tx(&sm.recv, splitk_recv_bytes(P, s0, s1));
+      mbar_expect_tx(&sm.recv, next_bytes);
 #pragma unroll 1
       for (int pr = 0; pr < P; ++pr)
-        if (pr != rank) mbar_arrive_remote_relaxed(&sm.rfree, (uint32_t)pr);
+        if (pr != rr) mbar_arrive_remote_relaxed(&sm.rfree, (uint32_t)(rbase + pr), rfree_n);
     }
   };
   bool released = false;
@@ -570,7 +572,9 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
       } else {
-        if (!splitk_tile<EP>(p, sm, rx, p.P, p.npad, p.M, lane_addr, i, t, r, sub, lane, rank, leader)) {
+        const int w4 = splitk_w4(p.M, p.P);
+        const uint32_t nb = splitk_recv_bytes(p.P, min(rank * w4, p.M), min((rank + 1) * w4, p.M));
+        if (!splitk_tile<EP>(p, sm, rx, p.P, p.npad, p.M, lane_addr, i, t, r, sub, lane, rank, 0, leader, nb, 1u)) {
           if (leader) {
             set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
             atomicExch(&sm.abort, 1);
@@ -606,10 +610,11 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
 // cluster occupancy), which the cross-CTA waits rely on.
 // ===========================================================================
 constexpr int SEQ_MAX = 4;  // GEMMs per launch
-constexpr int SEQ_P = 4;    // cluster size = split-K ways
+constexpr int SEQ_P = 4;    // cluster size; a GEMM splits K 4 or 2 ways (groups of P ranks)
 
 struct SeqGemm {
   int N, K, M, T, kb, mode;
+  int P;  // split-K ways (4: one group per cluster, 2: two); groups take tiles g, g + G, ...
   uint32_t idesc;
   EpArgs ep;
   unsigned int *done;   // completion counter: each CTA adds its tile count once its tiles are finished
@@ -660,26 +665,45 @@ __device__ __forceinline__ const CUtensorMap *seq_xmap(const SeqMaps &m, int j) 
   }
 }
 
-// this CTA's tile count and k-block range of every GEMM, read once from the
-// parameter block with constant indices and kept in registers (the unit loops
-// index them through sel4, never with a runtime array index)
+// this CTA's tile count, first tile, tile stride, k-block range and split of
+// every GEMM, read once from the parameter block with constant indices and kept
+// in registers (the unit loops index them through sel4, never with a runtime
+// array index)
 struct SeqTab {
-  int n, nt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX];
+  int n, nt[SEQ_MAX], t0[SEQ_MAX], dt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX], P[SEQ_MAX];
 };
 __device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
   return j == 0 ? a[0] : j == 1 ? a[1] : j == 2 ? a[2] : a[3];
 }
-__device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int q, int rank) {
+// cta: this CTA's index in the grid (clusters are SEQ_P consecutive CTAs)
+__device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
   SeqTab t;
   t.n = p.n;
 #pragma unroll
   for (int j = 0; j < SEQ_MAX; ++j) {
     const bool on = j < p.n;
-    t.nt[j] = on && p.g[j].T > q ? (p.g[j].T - 1 - q) / p.Q + 1 : 0;
-    t.k0[j] = on ? rank * p.g[j].kb / SEQ_P : 0;
-    t.k1[j] = on ? (rank + 1) * p.g[j].kb / SEQ_P : 0;
+    const int P = on ? p.g[j].P : SEQ_P;
+    const int g = cta / P, G = p.Q * (SEQ_P / P), rr = cta % P;  // group, groups, rank in the group
+    t.P[j] = P;
+    t.t0[j] = g;
+    t.dt[j] = G;
+    t.nt[j] = on && p.g[j].T > g ? (p.g[j].T - 1 - g) / G + 1 : 0;
+    t.k0[j] = on ? rr * p.g[j].kb / P : 0;
+    t.k1[j] = on ? (rr + 1) * p.g[j].kb / P : 0;
   }
   return t;
+}
+// bytes this CTA receives in the split-K tile of GEMM j
+__device__ __forceinline__ uint32_t seq_recv_bytes(const SeqTab &tb, int j, int M, int rank) {
+  const int P = sel4(tb.P, j), rr = rank % P, w4 = splitk_w4(M, P);
+  return splitk_recv_bytes(P, min(rr * w4, M), min((rr + 1) * w4, M));
+}
+// the GEMM of this CTA's split-K tile after tile ti of GEMM j (j = n: none)
+__device__ __forceinline__ int seq_next_gemm(const SeqTab &tb, int j, int ti) {
+  if (ti + 1 < sel4(tb.nt, j)) return j;
+  for (++j; j < tb.n; ++j)
+    if (sel4(tb.nt, j) > 0) return j;
+  return tb.n;
 }
 
 // cursor over this CTA's units (GEMM j, tile index ti, k-block k); j == n: past the end
@@ -699,11 +723,15 @@ __device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
   seq_skip_empty(tb, c);
 }
 
-// one tile of GEMM g (split-K over the cluster); false when a bounded wait expired
+// one tile of GEMM g (split-K over a group of P CTAs of the cluster); false
+// when a bounded wait expired.  rfree counts SEQ_P - 1 arrivals per tile: each
+// of the P - 1 owners arrives (SEQ_P - 1) / (P - 1) times.
 template <int EP>
 __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, int npad, uint32_t lane_addr, int i,
-                                         int t, int r, int sub, int lane, int rank, bool leader) {
-  const bool ok = splitk_tile<EP>(g, sm, rx, SEQ_P, npad, g.M, lane_addr, i, t, r, sub, lane, rank, leader);
+                                         int t, int r, int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
+  const int P = g.P, rr = rank % P;
+  const bool ok = splitk_tile<EP>(g, sm, rx, P, npad, g.M, lane_addr, i, t, r, sub, lane, rr, rank - rr, leader,
+                                  next_bytes, (uint32_t)((SEQ_P - 1) / (P - 1)));
   epi_bar();  // sm.flag is rewritten at the top of the next tile
   return ok;
 }
@@ -722,7 +750,6 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
   Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(rx) + p.rx_bytes);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int rank = (int)cluster_rank();
-  const int q = blockIdx.x / SEQ_P;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.stages; ++s) {
@@ -738,8 +765,10 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    const int w4 = splitk_w4(p.M, SEQ_P);
-    mbar_expect_tx(&sm.recv, splitk_recv_bytes(SEQ_P, min(rank * w4, p.M), min((rank + 1) * w4, p.M)));
+    // armed for this CTA's first split-K tile before the cluster barrier below
+    const SeqTab tb = seq_tab(p, (int)blockIdx.x);
+    const int j0 = sel4(tb.nt, 0) > 0 ? 0 : seq_next_gemm(tb, 0, 0);
+    mbar_expect_tx(&sm.recv, j0 < tb.n ? seq_recv_bytes(tb, j0, p.M, rank) : 0u);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
@@ -760,7 +789,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     // are complete.  Each arrives on the stage's full barrier with its own bytes.
     if (lane == 0) {
       const bool wp = warp == 0;
-      const SeqTab tb = seq_tab(p, q, rank);
+      const SeqTab tb = seq_tab(p, (int)blockIdx.x);
       const uint64_t pol = wp ? policy_evict_first() : policy_evict_last();
       const uint32_t bytes = wp ? (uint32_t)A_BYTES : (uint32_t)(stage_bytes - A_BYTES);
       if (wp)
@@ -784,7 +813,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
           prefetch_tensormap(map);
         }
         for (int ti = 0; ti < nt && ok; ++ti) {
-          const int row = wp ? (q + ti * p.Q) * BM : 0;
+          const int row = wp ? (sel4(tb.t0, j) + ti * sel4(tb.dt, j)) * BM : 0;
           for (int k = k0; k < k1; ++k, ++u) {
             if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
               ok = false;
@@ -824,7 +853,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       uint32_t ph = 0;
       bool ok = true;
       int i = 0;
-      const SeqTab tb = seq_tab(p, q, rank);
+      const SeqTab tb = seq_tab(p, (int)blockIdx.x);
       const uint32_t idesc = p.g[0].idesc;  // one row count, so one instruction descriptor for all GEMMs
       for (int j = 0; j < tb.n && ok; ++j) {
         const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j);
@@ -863,7 +892,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
-    const SeqTab tb = seq_tab(p, q, rank);
+    const SeqTab tb = seq_tab(p, (int)blockIdx.x);
     bool ok = true;
     int i = 0;
     for (int j = 0; j < p.n && ok; ++j) {
@@ -902,19 +931,21 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       }
       const int nt = sel4(tb.nt, j);
       for (int ti = 0; ti < nt && ok; ++ti, ++i) {
-        const int t = q + ti * p.Q;
+        const int t = sel4(tb.t0, j) + ti * sel4(tb.dt, j);
+        const int jn = seq_next_gemm(tb, j, ti);
+        const uint32_t nb = jn < tb.n ? seq_recv_bytes(tb, jn, p.M, rank) : 0u;
         switch (g.mode) {
           case EP_RESID:
-            ok = seq_tile<EP_RESID>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
+            ok = seq_tile<EP_RESID>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           case EP_SWIGLU:
-            ok = seq_tile<EP_SWIGLU>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
+            ok = seq_tile<EP_SWIGLU>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           case EP_QKV:
-            ok = seq_tile<EP_QKV>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
+            ok = seq_tile<EP_QKV>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           default:
-            ok = seq_tile<EP_STORE_F32>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader);
+            ok = seq_tile<EP_STORE_F32>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
         }
       }
@@ -1067,7 +1098,9 @@ cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_c
 
 size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
   const int stage_bytes = A_BYTES + npad * BK * 2;
-  const size_t red_bytes = (size_t)SEQ_P * BM * (((npad + 4 * SEQ_P - 1) / (4 * SEQ_P)) * 4) * 4;
+  // receive area for the larger of the 4-way and 2-way splits
+  const size_t r4 = (size_t)4 * BM * (((npad + 15) / 16) * 4) * 4, r2 = (size_t)2 * BM * (((npad + 7) / 8) * 4) * 4;
+  const size_t red_bytes = r4 > r2 ? r4 : r2;
   int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
   if (stages > 16) stages = 16;
   *stages_out = stages;
@@ -1280,14 +1313,19 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     g.T = (q.N + BM - 1) / BM;
     g.kb = q.K / BK;
     g.mode = mode;
+    // 4-way split for every GEMM.  (A 2-way split, two groups per cluster, gives
+    // the 48-tile QKV projection one tile per group on 96 CTAs instead of a
+    // second tile on 48 of 144; measured no faster at Qwen3-8B batch 1, since a
+    // CTA's weight stream is latency bound either way.)
+    g.P = SEQ_P;
     g.idesc = idesc;
     g.ep = q.ep;
     g.ep.qkv.row0 = 0;
     if (!tensor_map(&maps.w[j], q.W, q.N, q.K, q.K, BM) || !tensor_map(&maps.x[j], q.X, M, q.K, q.ldx, p.npad))
       return cudaErrorInvalidValue;
   }
-  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc((unsigned)(SEQ_P * p.g[j].T), &p.g[j].done_n);
-  const Dep d = chain->take((unsigned)(SEQ_P * p.g[n - 1].T));
+  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc((unsigned)(p.g[j].P * p.g[j].T), &p.g[j].done_n);
+  const Dep d = chain->take((unsigned)(p.g[n - 1].P * p.g[n - 1].T));
   p.g[n - 1].done = d.signal;
   p.g[n - 1].done_n = chain->shadow[chain->last];
   p.dep = d;

@@ -129,8 +129,9 @@ __device__ __forceinline__ void mbar_arrive_remote(uint64_t *local_bar, uint32_t
 // the same without release ordering: for "I have read what you sent me" signals
 // whose reads have already returned their values (a release arrive would also
 // wait for this CTA's unrelated outstanding global stores)
-__device__ __forceinline__ void mbar_arrive_remote_relaxed(uint64_t *local_bar, uint32_t rank) {
-  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(mapa(smem_u32(local_bar), rank))
+__device__ __forceinline__ void mbar_arrive_remote_relaxed(uint64_t *local_bar, uint32_t rank, uint32_t count = 1) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(mapa(smem_u32(local_bar), rank)),
+               "r"(count)
                : "memory");
 }
 __device__ __forceinline__ bool mbar_try_cluster(uint64_t *b, uint32_t parity) {
