@@ -43,6 +43,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--profile-only", action="store_true", help="warmup + a few steps, no timing legs (for ncu)")
+    p.add_argument("--depth", type=int, default=0,
+                   help="with --profile-only: target layers of a reduced-depth copy (same widths), for small ncu captures")
     return p.parse_args()
 
 
@@ -198,6 +200,22 @@ class OracleSample:
                 f"oracle's own calls")
 
 
+# DRAM bytes (read + write) per algorithmic byte of the persistent layer-segment
+# GEMM launch, from one ncu capture of it at Qwen3-8B widths and 17 rows
+# (dram__bytes_read.sum + dram__bytes_write.sum = 389.8 MB for 387.3 MB of
+# weights, activations and outputs).  Valid for that kernel as captured.
+SEQ_TRAFFIC_RATIO = {"qwen3_8b_b1": 1.006}
+
+
+def gemm_traffic(cfg, g):
+    """DRAM bytes of the mean GEMM launch of this run, scaled from the capture
+    (traffic grows with the weights streamed), or None without one."""
+    r = SEQ_TRAFFIC_RATIO.get(cfg.name)
+    if r is None or not g["launches"]:
+        return None
+    return round(r * g["bytes"] / g["launches"])
+
+
 def run_cpu_sample(cfg, steps: int, warmup: int, sched):
     s = OracleSample(cfg)
     for w in range(warmup):
@@ -283,6 +301,10 @@ def main():
         dist.barrier()
 
     cfg = synth.CONFIGS[args.config]
+    if args.depth:
+        assert args.profile_only, "--depth is for --profile-only captures"
+        cfg = cfg.replace(n_layers=args.depth, draft_layers=min(cfg.draft_layers, args.depth),
+                          feat_layers=tuple(sorted({1, args.depth})))
     K, Wm = args.steps, args.warmup
     n_rounds = Wm + K
     lens = synth.prompt_lengths(cfg)
@@ -398,7 +420,8 @@ def main():
                              "p50": round(float(np.percentile(per, 50)), 4),
                              "p90": round(float(np.percentile(per, 90)), 4)},
         "roofline": {"bound": "hbm", "achieved": round(gemm_gbs, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(gemm_gbs / hbm, 4), "traffic": None, "kernel": "weight-streaming GEMM",
+                     "frac": round(gemm_gbs / hbm, 4), "traffic": gemm_traffic(cfg, g),
+                     "kernel": "weight-streaming GEMM",
                      "peak_source": peak_src, "launches": g["launches"], "avg_launch_us": round(1e3 * g["ms"] / max(1, g["launches"]), 2)},
         "round_roofline": {"bound": "hbm", "alg_bytes": rb["total"], "achieved": round(round_gbs, 1), "peak": hbm,
                            "frac": round(round_gbs / hbm, 4), "unit": "GB/s", "peak_source": peak_src},
