@@ -65,7 +65,7 @@ struct Smem {
   uint32_t tmem;
   int flag;
   int abort;
-  float xch[16][64];
+  alignas(16) float xch[16][64];  // also the QKV epilogue's bf16 staging tile [16][128]
   float rv[4][16];
   int ri[4][16];
   float ssred[4][16];
@@ -87,13 +87,31 @@ __device__ __forceinline__ float silu_fast(float x) { return __fdividef(x, 1.0f 
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+// sums of x[0..15] over the warp's 32 lanes by recursive halving: at each step a
+// lane keeps half of its columns and adds the partner's copy of them, so 16
+// shuffles do the work of 16 butterfly reductions (80).  Returns the sum of
+// column (lane >> 1) & 15 (lanes 2c and 2c + 1 both hold column c).
+__device__ __forceinline__ float warp_column_sums16(const float *x, int lane) {
+  constexpr unsigned FULL = 0xffffffffu;
+  float a[8], b[4], c[2];
+  const bool h16 = lane & 16, h8 = lane & 8, h4 = lane & 4, h2 = lane & 2;
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    a[k] = (h16 ? x[k + 8] : x[k]) + __shfl_xor_sync(FULL, h16 ? x[k] : x[k + 8], 16);
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    b[k] = (h8 ? a[k + 4] : a[k]) + __shfl_xor_sync(FULL, h8 ? a[k] : a[k + 4], 8);
+#pragma unroll
+  for (int k = 0; k < 2; ++k)
+    c[k] = (h4 ? b[k + 2] : b[k]) + __shfl_xor_sync(FULL, h4 ? b[k] : b[k + 2], 4);
+  float d = (h2 ? c[1] : c[0]) + __shfl_xor_sync(FULL, h2 ? c[0] : c[1], 2);
+  return d + __shfl_xor_sync(FULL, d, 1);
+}
+
 // per-column sum over the tile's 128 rows (all epilogue threads call it)
 __device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const float *x, float *out) {
-#pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    const float t = warp_sum(x[j]);
-    if (lane == 0) sm.ssred[sub][j] = t;
-  }
+  const float d = warp_column_sums16(x, lane);
+  if (!(lane & 1)) sm.ssred[sub][(lane >> 1) & 15] = d;
   epi_bar();
 #pragma unroll
   for (int j = 0; j < 16; ++j) out[j] = sm.ssred[0][j] + sm.ssred[1][j] + sm.ssred[2][j] + sm.ssred[3][j];
@@ -102,14 +120,14 @@ __device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const f
 
 // prefetch of the inputs epilogue_chunk(t, c0, nc) will need (PT: any parameter
 // block with the GEMM's N, M and ep)
-template <int EP, typename PT>
+template <int EP, typename PT, int NC = 16>
 __device__ __forceinline__ void epilogue_prefetch(const PT &p, const Smem &sm, int t, int r, int c0, int nc,
                                                   EpPre &pre) {
   const EpArgs &ep = p.ep;
   const int n = t * BM + r, ncol = min(c0 + nc, p.M) - c0;
   if constexpr (EP == EP_RESID) {
 #pragma unroll
-    for (int j = 0; j < 16; ++j)
+    for (int j = 0; j < NC; ++j)
       pre.x[j] = (n < p.N && j < ncol) ? __ldcg(ep.out_f32 + (size_t)(c0 + j) * ep.ldo + n) : 0.f;
     pre.gain = (ep.out_xn != nullptr && n < p.N) ? ep.out_gain[n] : 0.f;
   } else if constexpr (EP == EP_QKV) {
@@ -117,130 +135,156 @@ __device__ __forceinline__ void epilogue_prefetch(const PT &p, const Smem &sm, i
     pre.gn = t < o.nq + o.hkv ? (t < o.nq ? o.qn : o.kn)[r] : 0.f;
     if (t < o.nq + o.hkv && r < 64) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j)
+      for (int j = 0; j < NC; ++j)
         pre.cs[j] = j < ncol ? o.rope[(size_t)sm.qkv_pos[c0 + j] * (BM / 2) + r] : make_float2(0.f, 0.f);
     }
   }
 }
 
-// epilogue on token columns c0 .. c0+nc-1 (nc <= 16) of tile t; v[j] = D[row r][c0+j]
-template <int EP, typename PT>
+// epilogue on token columns c0 .. c0+nc-1 (nc <= NC <= 16) of tile t; v[j] = D[row r][c0+j].
+// Every argument a loop needs is read into a register before the first store
+// (a store through a generic pointer could alias the parameter block, which
+// would make the compiler re-read it after each store).
+template <int EP, typename PT, int NC = 16>
 __device__ __forceinline__ void epilogue_chunk(const PT &p, Smem &sm, int t, int r, int sub, int lane, int c0,
                                                int nc, float *v, const EpPre &pre) {
+  static_assert(NC >= 1 && NC <= 16, "chunk width");
   const int n = t * BM + r;
   const EpArgs &ep = p.ep;
   const int cend = min(c0 + nc, p.M);
   if (ep.in_ss) {
 #pragma unroll
-    for (int j = 0; j < 16; ++j) v[j] *= sm.col_scale[min(c0 + j, MAX_NPAD - 1)];
+    for (int j = 0; j < NC; ++j) v[j] *= sm.col_scale[min(c0 + j, MAX_NPAD - 1)];
   }
   if constexpr (EP == EP_STORE_F32 || EP == EP_SILU) {
     if (n < p.N) {
+      float *const out_f32 = ep.out_f32 + n;
+      bf16 *const out_t = reinterpret_cast<bf16 *>(ep.out_t) + n;
+      const size_t ldo = ep.ldo, ldt = ep.ldt;
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
+      for (int j = 0; j < NC; ++j) {
         const int col = c0 + j;
         if (col < cend) {
-          if constexpr (EP == EP_STORE_F32) ep.out_f32[(size_t)col * ep.ldo + n] = v[j];
-          if constexpr (EP == EP_SILU)
-            reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + n] = __float2bfloat16_rn(silu_fast(v[j]));
+          if constexpr (EP == EP_STORE_F32) out_f32[(size_t)col * ldo] = v[j];
+          if constexpr (EP == EP_SILU) out_t[(size_t)col * ldt] = __float2bfloat16_rn(silu_fast(v[j]));
         }
       }
     }
   } else if constexpr (EP == EP_RESID) {
+    // arguments in registers before the first store (a store could alias them)
+    float *const out_f32 = ep.out_f32 + n;
+    bf16 *const out_xn = ep.out_xn ? reinterpret_cast<bf16 *>(ep.out_xn) + n : nullptr;
+    bf16 *const out_stash = ep.out_stash ? reinterpret_cast<bf16 *>(ep.out_stash) + n : nullptr;
+    float *const out_ss = ep.out_ss;
+    const size_t ldo = ep.ldo, ld_xn = ep.ld_xn, ld_stash = ep.ld_stash;
+    const int ld_ss = ep.ld_ss;
     float x[16];
-    const bool row_ok = n < p.N, has_xn = ep.out_xn != nullptr, has_stash = ep.out_stash != nullptr;
+    const bool row_ok = n < p.N, has_xn = out_xn != nullptr, has_stash = out_stash != nullptr;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
+    for (int j = NC; j < 16; ++j) x[j] = 0.f;
+#pragma unroll
+    for (int j = 0; j < NC; ++j) {
       const int col = c0 + j;
       x[j] = pre.x[j] + v[j];
       if (row_ok && col < cend) {
-        ep.out_f32[(size_t)col * ep.ldo + n] = x[j];
-        if (has_xn) reinterpret_cast<bf16 *>(ep.out_xn)[(size_t)col * ep.ld_xn + n] = __float2bfloat16_rn(x[j] * pre.gain);
-        if (has_stash) reinterpret_cast<bf16 *>(ep.out_stash)[(size_t)col * ep.ld_stash + n] = __float2bfloat16_rn(x[j]);
+        out_f32[(size_t)col * ldo] = x[j];
+        if (has_xn) out_xn[(size_t)col * ld_xn] = __float2bfloat16_rn(x[j] * pre.gain);
+        if (has_stash) out_stash[(size_t)col * ld_stash] = __float2bfloat16_rn(x[j]);
       } else {
         x[j] = 0.f;
       }
     }
-    if (ep.out_ss) {
+    if (out_ss) {
       // squared-norm partial of this tile's 128 features; thread r < 16 owns column c0 + r
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float tj = warp_sum(x[j] * x[j]);
-        if (lane == 0) sm.ssred[sub][j] = tj;
-      }
+      for (int j = 0; j < NC; ++j) x[j] *= x[j];
+      const float d = warp_column_sums16(x, lane);
+      if (!(lane & 1)) sm.ssred[sub][(lane >> 1) & 15] = d;
       epi_bar();
       if (r < 16 && c0 + r < cend)
-        ep.out_ss[(size_t)t * ep.ld_ss + c0 + r] = sm.ssred[0][r] + sm.ssred[1][r] + sm.ssred[2][r] + sm.ssred[3][r];
+        out_ss[(size_t)t * ld_ss + c0 + r] = sm.ssred[0][r] + sm.ssred[1][r] + sm.ssred[2][r] + sm.ssred[3][r];
       epi_bar();
     }
   } else if constexpr (EP == EP_QKV) {
+    // arguments in registers before the first store (a store could alias them)
     const QkvOut &o = ep.qkv;
-    const int head = t;
-    const int kind = head < o.nq ? 0 : (head < o.nq + o.hkv ? 1 : 2);  // q, k, v
-    const int kvh = kind == 1 ? head - o.nq : head - o.nq - o.hkv;
-    float y[16];
+    const int head = t, nq = o.nq, hkv = o.hkv, row0 = o.row0;
+    const int kind = head < nq ? 0 : (head < nq + hkv ? 1 : 2);  // q, k, v
+    const int kvh = kind == 1 ? head - nq : head - nq - hkv;
+    // the head's 128 values of token column c go to dst0 + off(c): q rows, the
+    // drafter's block K/V, or the column's slot in the paged pool (off < 0: none)
+    const bool paged = kind != 0 && o.bk == nullptr;
+    const long long rstride = kind == 0 ? (long long)o.hq_row * BM : (long long)hkv * BM;
+    bf16 *const dst0 = kind == 0 ? static_cast<bf16 *>(o.q_out) + (size_t)head * BM
+                       : !paged  ? static_cast<bf16 *>(kind == 1 ? o.bk : o.bv) + (size_t)kvh * BM
+                                 : static_cast<bf16 *>(o.pool) + (size_t)((kind == 1 ? 0 : hkv) + kvh) * o.page_size * BM;
+    const float eps = o.eps;
+    // the chunk's bf16 results, [16 columns][128 dims], in the exchange area
+    bf16 *const stage = reinterpret_cast<bf16 *>(&sm.xch[0][0]);
     if (kind != 2) {
       // per-head RMSNorm over the 128 rows of the column, then rotary on pairs (r, r + 64)
-      float sq[16], tot[16];
+      float sq[16], tot[16], y[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) sq[j] = v[j] * v[j];
+      for (int j = 0; j < 16; ++j) sq[j] = j < NC ? v[j] * v[j] : 0.f;
       column_sums(sm, sub, lane, sq, tot);
       const float gn = pre.gn;
 #pragma unroll
-      for (int j = 0; j < 16; ++j) y[j] = v[j] * rsqrtf(tot[j] * (1.0f / BM) + o.eps) * gn;
+      for (int j = 0; j < NC; ++j) y[j] = v[j] * rsqrtf(tot[j] * (1.0f / BM) + eps) * gn;
       if (r >= 64) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) sm.xch[j][r - 64] = y[j];
+        for (int j = 0; j < NC; ++j) sm.xch[j][r - 64] = y[j];
       }
       epi_bar();
-    } else {
+      uint32_t lohi[16];  // bf16 pair (dim r, dim r + 64)
+      if (r < 64) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) y[j] = v[j];
-    }
-    if (kind == 2 || r < 64) {
-      // destinations: q rows, the drafter's block K/V, or the column's slot in the paged pool
-      const size_t kv_off = (size_t)((kind == 1 ? 0 : o.hkv) + kvh) * o.page_size * BM;
-#pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const int col = c0 + j;
-        const int grow = o.row0 + col;
-        bf16 *dst;
-        bool wr = col < cend;
-        if (kind == 0) {
-          dst = static_cast<bf16 *>(o.q_out) + ((size_t)grow * o.hq_row + head) * BM;
-        } else if (o.bk != nullptr) {
-          dst = static_cast<bf16 *>(kind == 1 ? o.bk : o.bv) + ((size_t)grow * o.hkv + kvh) * BM;
-        } else {
-          const long long base = wr ? sm.qkv_base[col] : -1;
-          wr = base >= 0;
-          dst = static_cast<bf16 *>(o.pool) + (wr ? (size_t)base + kv_off : 0);
-        }
-        if (!wr) continue;
-        if (kind == 2) {
-          dst[r] = __float2bfloat16_rn(y[j]);
-        } else {
+        for (int j = 0; j < NC; ++j) {
           const float2 cs = pre.cs[j];
           const float x1 = y[j], x2 = sm.xch[j][r];
-          dst[r] = __float2bfloat16_rn(x1 * cs.x - x2 * cs.y);
-          dst[r + 64] = __float2bfloat16_rn(x2 * cs.x + x1 * cs.y);
+          const __nv_bfloat162 b2 = __floats2bfloat162_rn(x1 * cs.x - x2 * cs.y, x2 * cs.x + x1 * cs.y);
+          lohi[j] = *reinterpret_cast<const uint32_t *>(&b2);
         }
       }
+      epi_bar();  // every read of the exchange area is done before it becomes the staging tile
+      if (r < 64) {
+#pragma unroll
+        for (int j = 0; j < NC; ++j) {
+          const __nv_bfloat162 b2 = *reinterpret_cast<const __nv_bfloat162 *>(&lohi[j]);
+          stage[j * BM + r] = b2.x;
+          stage[j * BM + r + 64] = b2.y;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < NC; ++j) stage[j * BM + r] = __float2bfloat16_rn(v[j]);
     }
-    if (kind != 2) epi_bar();  // xch is rewritten by the next chunk
+    epi_bar();
+    // 16-byte stores: vector e holds dims 8 (e % 16) .. of column c0 + e / 16
+    const int nv = (cend - c0) * 16;
+    for (int e = r; e < nv; e += BM) {
+      const int jc = e >> 4, part = e & 15, col = c0 + jc;
+      const long long off = paged ? sm.qkv_base[col] : (long long)(row0 + col) * rstride;
+      if (off >= 0)
+        *reinterpret_cast<uint4 *>(dst0 + off + part * 8) = *reinterpret_cast<const uint4 *>(stage + jc * BM + part * 8);
+    }
+    epi_bar();  // the staging tile is rewritten by the next chunk
   } else if constexpr (EP == EP_SWIGLU) {
     // rows 0..63 of the tile are gate features 64t.., rows 64..127 the matching up features
+    bf16 *const out_t = reinterpret_cast<bf16 *>(ep.out_t) + t * 64 + r;
+    const size_t ldt = ep.ldt;
     if (r >= 64) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) sm.xch[j][r - 64] = v[j];
+      for (int j = 0; j < NC; ++j) sm.xch[j][r - 64] = v[j];
     }
     epi_bar();
     if (r < 64 && t * BM + 64 + r < p.N) {
+      float up[NC];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
+      for (int j = 0; j < NC; ++j) up[j] = sm.xch[j][r];
+#pragma unroll
+      for (int j = 0; j < NC; ++j) {
         const int col = c0 + j;
-        if (col < cend)
-          reinterpret_cast<bf16 *>(ep.out_t)[(size_t)col * ep.ldt + t * 64 + r] =
-              __float2bfloat16_rn(silu_fast(v[j]) * sm.xch[j][r]);
+        if (col < cend) out_t[(size_t)col * ldt] = __float2bfloat16_rn(silu_fast(v[j]) * up[j]);
       }
     }
     epi_bar();
@@ -262,9 +306,12 @@ __device__ __forceinline__ void epilogue_chunk(const PT &p, Smem &sm, int t, int
 #pragma unroll
       for (int s = 1; s < 4; ++s) argmax_merge(bv, bi, sm.rv[s][lane], sm.ri[s][lane]);
       const int col = c0 + lane;
+      float *const part_val = ep.part_val;
+      int *const part_idx = ep.part_idx;
+      const size_t n_tiles = ep.n_tiles;
       if (col < cend) {
-        ep.part_val[(size_t)col * ep.n_tiles + t] = bv;
-        ep.part_idx[(size_t)col * ep.n_tiles + t] = bi;
+        part_val[(size_t)col * n_tiles + t] = bv;
+        part_idx[(size_t)col * n_tiles + t] = bi;
       }
     }
     epi_bar();
@@ -294,15 +341,21 @@ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
 // runs the fused epilogue.  It re-arms recv with next_bytes (what its next
 // split-K tile will receive) before telling the senders (rfree, rfree_n
 // arrivals each) that they may push again.  False when a wait expired.
-template <int EP, typename PT>
-__device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P, int npad, int M,
+// CW4 > 0: the split is 4-way over npad = 4 CW4 columns (each owner finishes
+// CW4 of them), known at compile time: every loop has a fixed trip count, the
+// owner of a column group is a constant, and the epilogue covers CW4 columns.
+template <int EP, typename PT, int CW4 = 0>
+__device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P_, int npad_, int M,
                                             uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
                                             int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n) {
-  const int w4 = splitk_w4(M, P);
+  static_assert(CW4 % 4 == 0 && CW4 <= 16, "owner width");
+  constexpr int NC = CW4 ? CW4 : 16;  // epilogue columns per chunk
+  const int P = CW4 ? 4 : P_, npad = CW4 ? 4 * CW4 : npad_;
+  const int w4 = CW4 ? CW4 : splitk_w4(M, P);
   const int s0 = min(rr * w4, M), s1 = min((rr + 1) * w4, M);
   const int buf = i & 1;
   EpPre pre;
-  epilogue_prefetch<EP>(g, sm, t, r, s0, min(16, s1 - s0), pre);
+  epilogue_prefetch<EP, PT, NC>(g, sm, t, r, s0, min(NC, s1 - s0), pre);
   if (leader) {
     int ok = mbar_wait(&sm.accf[buf], (i >> 1) & 1) ? 1 : 0;
     if (ok && i > 0) ok = mbar_wait_cluster(&sm.rfree, (i - 1) & 1) ? 1 : 0;
@@ -315,7 +368,8 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
   const uint32_t acc_addr = lane_addr + buf * npad;
   const uint32_t rx_s = smem_u32(rx), recv_s = smem_u32(&sm.recv);
   float v[16];
-  for (int c0 = 0; c0 < npad && c0 < M; c0 += 16) {
+  // the row's partial of columns c0 .. c0 + 15, pushed group by group to the groups' owners
+  auto push16 = [&](int c0) {
     tmem_ld16(acc_addr + c0, v);
 #pragma unroll
     for (int q4 = 0; q4 < 4; ++q4) {
@@ -329,6 +383,13 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
       else
         st_async_f4(mapa(rx_s + (uint32_t)e * 4, (uint32_t)(rbase + owner)), x, mapa(recv_s, (uint32_t)(rbase + owner)));
     }
+  };
+  if constexpr (CW4 > 0) {
+#pragma unroll
+    for (int c0 = 0; c0 < 4 * CW4; c0 += 16)
+      if (c0 < M) push16(c0);
+  } else {
+    for (int c0 = 0; c0 < npad && c0 < M; c0 += 16) push16(c0);
   }
   tc_fence_before();
   __syncwarp();
@@ -354,10 +415,11 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
     for (int c0 = s0; c0 < s1; c0 += 16) {
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = 0.f;
-      for (int sp = 0; sp < P; ++sp) {
+      // the P partials of the row, in rank order
+      auto add_partial = [&](int sp) {
         const float *src = rx + (sp * BM + r) * w4 + (c0 - s0);
 #pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
+        for (int q4 = 0; q4 < NC / 4; ++q4) {
           if (c0 + 4 * q4 >= s1) break;
           const float4 y = *reinterpret_cast<const float4 *>(src + 4 * q4);
           v[4 * q4] += y.x;
@@ -365,13 +427,19 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
           v[4 * q4 + 2] += y.z;
           v[4 * q4 + 3] += y.w;
         }
+      };
+      if constexpr (CW4 > 0) {
+#pragma unroll
+        for (int sp = 0; sp < 4; ++sp) add_partial(sp);
+      } else {
+        for (int sp = 0; sp < P; ++sp) add_partial(sp);
       }
       if (c0 + 16 >= s1) {
         release();
         released = true;
       }
-      if (c0 > s0) epilogue_prefetch<EP>(g, sm, t, r, c0, min(16, s1 - c0), pre);
-      epilogue_chunk<EP>(g, sm, t, r, sub, lane, c0, min(16, s1 - c0), v, pre);
+      if (c0 > s0) epilogue_prefetch<EP, PT, NC>(g, sm, t, r, c0, min(NC, s1 - c0), pre);
+      epilogue_chunk<EP, PT, NC>(g, sm, t, r, sub, lane, c0, min(NC, s1 - c0), v, pre);
     }
   }
   if (!released) release();
@@ -723,21 +791,24 @@ __device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
   seq_skip_empty(tb, c);
 }
 
-// one tile of GEMM g (split-K over a group of P CTAs of the cluster); false
-// when a bounded wait expired.  rfree counts SEQ_P - 1 arrivals per tile: each
-// of the P - 1 owners arrives (SEQ_P - 1) / (P - 1) times.
-template <int EP>
-__device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, int npad, uint32_t lane_addr, int i,
-                                         int t, int r, int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
-  const int P = g.P, rr = rank % P;
-  const bool ok = splitk_tile<EP>(g, sm, rx, P, npad, g.M, lane_addr, i, t, r, sub, lane, rr, rank - rr, leader,
-                                  next_bytes, (uint32_t)((SEQ_P - 1) / (P - 1)));
+// one tile of GEMM g (split-K over the SEQ_P CTAs of the cluster, NPAD token
+// columns); false when a bounded wait expired.  rfree counts SEQ_P - 1
+// arrivals per tile, one from each other owner.
+template <int EP, int NPAD>
+__device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, uint32_t lane_addr, int i, int t, int r,
+                                         int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
+  static_assert(SEQ_P == 4, "the compile-time split of splitk_tile is 4-way");
+  const bool ok = splitk_tile<EP, SeqGemm, NPAD / 4>(g, sm, rx, SEQ_P, NPAD, g.M, lane_addr, i, t, r, sub, lane, rank, 0,
+                                                     leader, next_bytes, 1u);
   epi_bar();  // sm.flag is rewritten at the top of the next tile
   return ok;
 }
 
 constexpr int SEQ_THREADS = THREADS + 32;  // warp 6: the activation producer
 
+// NPAD: the token columns padded to 16 (p.npad), a compile-time constant so that
+// the split-K epilogue has fixed trip counts
+template <int NPAD>
 __global__ void __launch_bounds__(SEQ_THREADS, 1)
 k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqParams p) {
   // the next launch may start once every CTA of this one runs; it waits on the
@@ -936,16 +1007,16 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         const uint32_t nb = jn < tb.n ? seq_recv_bytes(tb, jn, p.M, rank) : 0u;
         switch (g.mode) {
           case EP_RESID:
-            ok = seq_tile<EP_RESID>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           case EP_SWIGLU:
-            ok = seq_tile<EP_SWIGLU>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_SWIGLU, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           case EP_QKV:
-            ok = seq_tile<EP_QKV>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
           default:
-            ok = seq_tile<EP_STORE_F32>(g, sm, rx, p.npad, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
             break;
         }
       }
@@ -1098,9 +1169,8 @@ cudaError_t run(const CUtensorMap &mw, const CUtensorMap &mx, Params p, int sm_c
 
 size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
   const int stage_bytes = A_BYTES + npad * BK * 2;
-  // receive area for the larger of the 4-way and 2-way splits
-  const size_t r4 = (size_t)4 * BM * (((npad + 15) / 16) * 4) * 4, r2 = (size_t)2 * BM * (((npad + 7) / 8) * 4) * 4;
-  const size_t red_bytes = r4 > r2 ? r4 : r2;
+  // receive area of the 4-way split: a [BM][npad / 4] fp32 slot per rank
+  const size_t red_bytes = (size_t)SEQ_P * BM * (npad / SEQ_P) * 4;
   int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
   if (stages > 16) stages = 16;
   *stages_out = stages;
@@ -1109,14 +1179,27 @@ size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
 }
 
 // clusters of SEQ_P persistent CTAs that are resident at once
-int seq_clusters(size_t smem) {
+using SeqKernel = void (*)(SeqMaps, SeqParams);
+// the instantiation for npad token columns (16, 32, 48 or 64), or null
+SeqKernel seq_kernel(int npad) {
+  switch (npad) {
+    case 16: return k_gemm_seq<16>;
+    case 32: return k_gemm_seq<32>;
+    case 48: return k_gemm_seq<48>;
+    case 64: return k_gemm_seq<64>;
+    default: return nullptr;
+  }
+}
+
+int seq_clusters(int npad, size_t smem) {
   static std::mutex mu;
-  static std::map<size_t, int> cache;
+  static std::map<std::pair<int, size_t>, int> cache;
   std::lock_guard<std::mutex> lock(mu);
-  auto it = cache.find(smem);
+  auto it = cache.find({npad, smem});
   if (it != cache.end()) return it->second;
   int n = 0;
-  if (cudaFuncSetAttribute(k_gemm_seq, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048) ==
+  const SeqKernel kern = seq_kernel(npad);
+  if (kern && cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048) ==
       cudaSuccess) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(SEQ_P);
@@ -1129,10 +1212,10 @@ int seq_clusters(size_t smem) {
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    if (cudaOccupancyMaxActiveClusters(&n, k_gemm_seq, &cfg) != cudaSuccess) n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
   }
   cudaGetLastError();
-  cache.emplace(smem, n);
+  cache.emplace(std::make_pair(npad, smem), n);
   return n;
 }
 
@@ -1297,7 +1380,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   while (cols < 2 * p.npad) cols <<= 1;
   p.tmem_cols = cols;
   const size_t smem = seq_smem(p.npad, &p.stages, &p.rx_bytes);
-  p.Q = seq_clusters(smem);
+  p.Q = seq_clusters(p.npad, smem);
   if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
   const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   for (int j = 0; j < n; ++j) {
@@ -1345,7 +1428,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   at[1].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k_gemm_seq, maps, p);
+  return cudaLaunchKernelEx(&cfg, seq_kernel(p.npad), maps, p);
 }
 
 }  // namespace dflow
