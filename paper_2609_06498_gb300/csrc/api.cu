@@ -987,7 +987,9 @@ dflow_status check_call(dflow_handle *h, const dflow_state *st) {
 Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
   DepChain &d = h->dep;
   if (d.dirty && d.dev != nullptr) {
-    if (cudaMemsetAsync(d.dev, 0, kDepSlots * sizeof(unsigned int), (cudaStream_t)stream) == cudaSuccess) {
+    // with the counters, the persistent GEMM's leftover sums (a failed launch may have left partials)
+    if (cudaMemsetAsync(d.dev, 0, kDepSlots * sizeof(unsigned int), (cudaStream_t)stream) == cudaSuccess &&
+        (!h->use_tc || tc_init(h->tcw, (cudaStream_t)stream) == cudaSuccess)) {
       for (int i = 0; i < kDepSlots; ++i) d.shadow[i] = 0;
       d.next = 0;
       d.dirty = false;

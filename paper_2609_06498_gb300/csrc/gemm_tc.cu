@@ -65,6 +65,7 @@ struct Smem {
   uint32_t tmem;
   int flag;
   int abort;
+  int left_last;  // the leftover part just finished completed its columns' count
   alignas(16) float xch[16][64];  // also the QKV epilogue's bf16 staging tile [16][128]
   float rv[4][16];
   int ri[4][16];
@@ -331,6 +332,23 @@ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
   return s1 > s0 ? (uint32_t)((P - 1) * BM * ((s1 - s0 + 3) / 4) * 16) : 0u;
 }
 
+// A cluster's part of a tile that several clusters share: the fp32 sums of the
+// tile [BM][npad], the arrival count of this CTA's columns, and the parts.
+struct LeftPart {
+  float *acc = nullptr;
+  unsigned int *ctr = nullptr;
+  unsigned int parts = 0;
+};
+__device__ __forceinline__ void red_add_v4(float *a, float x, float y, float z, float w) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(a), "f"(x), "f"(y), "f"(z), "f"(w) : "memory");
+}
+__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
+__device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsigned int v) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+  return old;
+}
+
 // One tile of a P-way split-K GEMM (P > 1) done by the P CTAs at cluster ranks
 // rbase .. rbase + P - 1 (this CTA is the rr-th).  Every one holds a partial of
 // the whole [128 x M] tile; the rr-th finishes token columns [s0, s1).
@@ -345,9 +363,13 @@ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
 // CW4 of them), known at compile time: every loop has a fixed trip count, the
 // owner of a column group is a constant, and the epilogue covers CW4 columns.
 template <int EP, typename PT, int CW4 = 0>
+// lp.acc set (CW4 > 0 only): the cluster holds one part of the tile; each owner
+// adds its columns' sum into lp.acc and only the one completing the count runs
+// their epilogue (sm.left_last = 1 in that CTA).
 __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P_, int npad_, int M,
                                             uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
-                                            int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n) {
+                                            int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n,
+                                            const LeftPart lp = LeftPart{}) {
   static_assert(CW4 % 4 == 0 && CW4 <= 16, "owner width");
   constexpr int NC = CW4 ? CW4 : 16;  // epilogue columns per chunk
   const int P = CW4 ? 4 : P_, npad = CW4 ? 4 * CW4 : npad_;
@@ -439,6 +461,33 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
         released = true;
       }
       if (c0 > s0) epilogue_prefetch<EP, PT, NC>(g, sm, t, r, c0, min(NC, s1 - c0), pre);
+      if constexpr (CW4 > 0) {
+        if (lp.acc != nullptr) {
+          // one chunk (CW4 <= 16): this cluster's part of the columns into the tile's sums
+          float *const a = lp.acc + (size_t)r * npad + c0;
+#pragma unroll
+          for (int q4 = 0; q4 < NC / 4; ++q4)
+            if (c0 + 4 * q4 < s1) red_add_v4(a + 4 * q4, v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+          fence_acq_rel_gpu();  // this thread's additions are visible before the count below
+          epi_bar();
+          if (leader) sm.left_last = atom_add_acq_rel(lp.ctr, 1u) == lp.parts - 1 ? 1 : 0;
+          epi_bar();
+          if (!sm.left_last) continue;
+          // every part is in (the leader's acquire, ordered before these reads by the barrier):
+          // the sums, leaving zeros for the next use
+#pragma unroll
+          for (int q4 = 0; q4 < NC / 4; ++q4) {
+            if (c0 + 4 * q4 >= s1) break;
+            const float4 x = __ldcg(reinterpret_cast<const float4 *>(a + 4 * q4));
+            __stcg(reinterpret_cast<float4 *>(a + 4 * q4), make_float4(0.f, 0.f, 0.f, 0.f));
+            v[4 * q4] = x.x;
+            v[4 * q4 + 1] = x.y;
+            v[4 * q4 + 2] = x.z;
+            v[4 * q4 + 3] = x.w;
+          }
+          if (leader) *reinterpret_cast<volatile unsigned int *>(lp.ctr) = 0u;
+        }
+      }
       epilogue_chunk<EP, PT, NC>(g, sm, t, r, sub, lane, c0, min(NC, s1 - c0), v, pre);
     }
   }
@@ -678,15 +727,26 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
 // cluster occupancy), which the cross-CTA waits rely on.
 // ===========================================================================
 constexpr int SEQ_MAX = 4;  // GEMMs per launch
-constexpr int SEQ_P = 4;    // cluster size; a GEMM splits K 4 or 2 ways (groups of P ranks)
+constexpr int SEQ_P = 4;    // cluster size = split-K ways of a tile inside a cluster
+constexpr int SEQ_LEFT_MAX = 40;  // leftover tiles of one GEMM (fewer than the clusters, at most 38)
 
+// Tiles 0 .. Tf-1 go to the Q clusters round robin (cluster q: q, q + Q, ...),
+// each split 4 ways over the cluster's CTAs and reduced in shared memory.  The
+// Tl = T - Tf leftover tiles (T mod Q of them, when Q is a multiple) are each
+// split over ls = Q / Tl clusters, 4 ls ways: every CTA then streams the same
+// number of weight k-blocks.  A cluster reduces its part of a leftover tile in
+// shared memory like any tile; each column owner then adds its columns in fp32
+// into lacc (L2), and the owner whose addition completes the count of its
+// columns runs their epilogue and leaves lacc and the count at zero again.
 struct SeqGemm {
   int N, K, M, T, kb, mode;
-  int P;  // split-K ways (4: one group per cluster, 2: two); groups take tiles g, g + G, ...
+  int Tf, Tl, ls;
   uint32_t idesc;
   EpArgs ep;
-  unsigned int *done;   // completion counter: each CTA adds its tile count once its tiles are finished
+  unsigned int *done;   // completion counter: each CTA adds 1 per tile whose columns it finished
   unsigned int done_n;  // its value once every tile of this GEMM is finished
+  float *lacc;          // [Tl][BM][npad] leftover sums (zero between uses)
+  unsigned int *lctr;   // [Tl][SEQ_P] leftover contributions per column owner (zero between uses)
 };
 struct SeqMaps {
   CUtensorMap w[SEQ_MAX], x[SEQ_MAX];  // weights [N][K], activations [M][K]
@@ -738,7 +798,8 @@ __device__ __forceinline__ const CUtensorMap *seq_xmap(const SeqMaps &m, int j) 
 // in registers (the unit loops index them through sel4, never with a runtime
 // array index)
 struct SeqTab {
-  int n, nt[SEQ_MAX], t0[SEQ_MAX], dt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX], P[SEQ_MAX];
+  int n, nt[SEQ_MAX], t0[SEQ_MAX], dt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX];
+  int lt[SEQ_MAX], lk0[SEQ_MAX], lk1[SEQ_MAX];  // leftover tile (index among the leftovers, or -1) and k range
 };
 __device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
   return j == 0 ? a[0] : j == 1 ? a[1] : j == 2 ? a[2] : a[3];
@@ -747,59 +808,53 @@ __device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
 __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
   SeqTab t;
   t.n = p.n;
+  const int q = cta / SEQ_P, rr = cta % SEQ_P;  // cluster, rank in the cluster
 #pragma unroll
   for (int j = 0; j < SEQ_MAX; ++j) {
     const bool on = j < p.n;
-    const int P = on ? p.g[j].P : SEQ_P;
-    const int g = cta / P, G = p.Q * (SEQ_P / P), rr = cta % P;  // group, groups, rank in the group
-    t.P[j] = P;
-    t.t0[j] = g;
-    t.dt[j] = G;
-    t.nt[j] = on && p.g[j].T > g ? (p.g[j].T - 1 - g) / G + 1 : 0;
-    t.k0[j] = on ? rr * p.g[j].kb / P : 0;
-    t.k1[j] = on ? (rr + 1) * p.g[j].kb / P : 0;
+    const int kb = on ? p.g[j].kb : 0, Tf = on ? p.g[j].Tf : 0, Tl = on ? p.g[j].Tl : 0, ls = on ? p.g[j].ls : 1;
+    t.t0[j] = q;
+    t.dt[j] = p.Q;
+    t.nt[j] = Tf > q ? (Tf - 1 - q) / p.Q + 1 : 0;
+    t.k0[j] = rr * kb / SEQ_P;
+    t.k1[j] = (rr + 1) * kb / SEQ_P;
+    const bool left = q < Tl * ls;
+    const int m = (q % ls) * SEQ_P + rr, parts = SEQ_P * ls;  // this CTA's part of its leftover tile
+    t.lt[j] = left ? q / ls : -1;
+    t.lk0[j] = left ? m * kb / parts : 0;
+    t.lk1[j] = left ? (m + 1) * kb / parts : 0;
   }
   return t;
 }
-// bytes this CTA receives in the split-K tile of GEMM j
-__device__ __forceinline__ uint32_t seq_recv_bytes(const SeqTab &tb, int j, int M, int rank) {
-  const int P = sel4(tb.P, j), rr = rank % P, w4 = splitk_w4(M, P);
-  return splitk_recv_bytes(P, min(rr * w4, M), min((rr + 1) * w4, M));
+// bytes this CTA receives in a split-K tile of GEMM j
+__device__ __forceinline__ uint32_t seq_recv_bytes(int M, int rank) {
+  const int w4 = splitk_w4(M, SEQ_P);
+  return splitk_recv_bytes(SEQ_P, min(rank * w4, M), min((rank + 1) * w4, M));
 }
-// the GEMM of this CTA's split-K tile after tile ti of GEMM j (j = n: none)
-__device__ __forceinline__ int seq_next_gemm(const SeqTab &tb, int j, int ti) {
-  if (ti + 1 < sel4(tb.nt, j)) return j;
+// true when this CTA has another tile after tile ti of GEMM j (ti = -1: its leftover part)
+__device__ __forceinline__ bool seq_more(const SeqTab &tb, int j, int ti) {
+  if (ti + 1 < sel4(tb.nt, j)) return true;
   for (++j; j < tb.n; ++j)
-    if (sel4(tb.nt, j) > 0) return j;
-  return tb.n;
-}
-
-// cursor over this CTA's units (GEMM j, tile index ti, k-block k); j == n: past the end
-struct SeqCur {
-  int j, ti, k;
-};
-__device__ __forceinline__ void seq_skip_empty(const SeqTab &tb, SeqCur &c) {
-  while (c.j < tb.n && sel4(tb.nt, c.j) == 0) ++c.j;
-  c.ti = 0;
-  if (c.j < tb.n) c.k = sel4(tb.k0, c.j);
-}
-__device__ __forceinline__ void seq_next(const SeqTab &tb, SeqCur &c) {
-  if (++c.k < sel4(tb.k1, c.j)) return;
-  c.k = sel4(tb.k0, c.j);
-  if (++c.ti < sel4(tb.nt, c.j)) return;
-  ++c.j;
-  seq_skip_empty(tb, c);
+    if (sel4(tb.nt, j) > 0 || sel4(tb.lt, j) >= 0) return true;
+  return false;
 }
 
 // one tile of GEMM g (split-K over the SEQ_P CTAs of the cluster, NPAD token
 // columns); false when a bounded wait expired.  rfree counts SEQ_P - 1
 // arrivals per tile, one from each other owner.
+// lt >= 0: t is leftover tile lt, the cluster holds one part of it.
 template <int EP, int NPAD>
-__device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, uint32_t lane_addr, int i, int t, int r,
-                                         int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
+__device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, uint32_t lane_addr, int i, int t, int lt,
+                                         int r, int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
   static_assert(SEQ_P == 4, "the compile-time split of splitk_tile is 4-way");
+  LeftPart lp;
+  if (lt >= 0) {
+    lp.acc = g.lacc + (size_t)lt * BM * NPAD;
+    lp.ctr = g.lctr + lt * SEQ_P + rank;
+    lp.parts = (unsigned int)g.ls;
+  }
   const bool ok = splitk_tile<EP, SeqGemm, NPAD / 4>(g, sm, rx, SEQ_P, NPAD, g.M, lane_addr, i, t, r, sub, lane, rank, 0,
-                                                     leader, next_bytes, 1u);
+                                                     leader, next_bytes, 1u, lp);
   epi_bar();  // sm.flag is rewritten at the top of the next tile
   return ok;
 }
@@ -838,8 +893,9 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // armed for this CTA's first split-K tile before the cluster barrier below
     const SeqTab tb = seq_tab(p, (int)blockIdx.x);
-    const int j0 = sel4(tb.nt, 0) > 0 ? 0 : seq_next_gemm(tb, 0, 0);
-    mbar_expect_tx(&sm.recv, j0 < tb.n ? seq_recv_bytes(tb, j0, p.M, rank) : 0u);
+    bool any = false;
+    for (int j = 0; j < tb.n; ++j) any = any || sel4(tb.nt, j) > 0 || sel4(tb.lt, j) >= 0;
+    mbar_expect_tx(&sm.recv, any ? seq_recv_bytes(p.M, rank) : 0u);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
@@ -869,8 +925,8 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       uint32_t ph = 0;
       bool ok = true;
       for (int j = 0; j < tb.n && ok; ++j) {
-        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j);
-        if (nt == 0) continue;
+        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j), lt = sel4(tb.lt, j);
+        if (nt == 0 && lt < 0) continue;
         const CUtensorMap *map = wp ? seq_wmap(maps, j) : seq_xmap(maps, j);
         if (!wp) {
           // GEMM j reads what GEMM j - 1 (or the previous launch) wrote
@@ -883,9 +939,12 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
           if (j > 0 || p.dep.wait) fence_proxy_async_global();
           prefetch_tensormap(map);
         }
-        for (int ti = 0; ti < nt && ok; ++ti) {
-          const int row = wp ? (sel4(tb.t0, j) + ti * sel4(tb.dt, j)) * BM : 0;
-          for (int k = k0; k < k1; ++k, ++u) {
+        // the leftover part first, then the full tiles
+        for (int ti = lt >= 0 ? -1 : 0; ti < nt && ok; ++ti) {
+          const int tile = ti < 0 ? p.g[j].Tf + lt : sel4(tb.t0, j) + ti * sel4(tb.dt, j);
+          const int row = wp ? tile * BM : 0;
+          const int kb0 = ti < 0 ? sel4(tb.lk0, j) : k0, kb1 = ti < 0 ? sel4(tb.lk1, j) : k1;
+          for (int k = kb0; k < kb1; ++k, ++u) {
             if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
               ok = false;
               break;
@@ -927,19 +986,20 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       const SeqTab tb = seq_tab(p, (int)blockIdx.x);
       const uint32_t idesc = p.g[0].idesc;  // one row count, so one instruction descriptor for all GEMMs
       for (int j = 0; j < tb.n && ok; ++j) {
-        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j);
-        for (int ti = 0; ti < nt && ok; ++ti, ++i) {
+        const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j), lt = sel4(tb.lt, j);
+        for (int ti = lt >= 0 ? -1 : 0; ti < nt && ok; ++ti, ++i) {
           const int buf = i & 1;
+          const int kb0 = ti < 0 ? sel4(tb.lk0, j) : k0, kb1 = ti < 0 ? sel4(tb.lk1, j) : k1;
           if (!mbar_wait(&sm.acce[buf], ((i >> 1) & 1) ^ 1)) { ok = false; break; }
           tc_fence_after();
           const uint32_t d = tmem + buf * p.npad;
-          for (int k = k0; k < k1; ++k) {
+          for (int k = kb0; k < kb1; ++k) {
             if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
             tc_fence_after();
             const uint32_t a = smem_u32(ring + (size_t)stage * stage_bytes);
             const uint64_t ad = smem_desc(a), bd = smem_desc(a + A_BYTES);
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (k > k0 || kk > 0) ? 1u : 0u);
+            for (int kk = 0; kk < BK / 16; ++kk) mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (k > kb0 || kk > 0) ? 1u : 0u);
             mma_commit(&sm.empty[stage]);
             if (++stage == p.stages) {
               stage = 0;
@@ -1000,28 +1060,31 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         }
         epi_bar();
       }
-      const int nt = sel4(tb.nt, j);
-      for (int ti = 0; ti < nt && ok; ++ti, ++i) {
-        const int t = sel4(tb.t0, j) + ti * sel4(tb.dt, j);
-        const int jn = seq_next_gemm(tb, j, ti);
-        const uint32_t nb = jn < tb.n ? seq_recv_bytes(tb, jn, p.M, rank) : 0u;
+      const int nt = sel4(tb.nt, j), lt = sel4(tb.lt, j);
+      unsigned int finished = 0;  // tiles whose columns of this CTA are written
+      for (int ti = lt >= 0 ? -1 : 0; ti < nt && ok; ++ti, ++i) {
+        const int t = ti < 0 ? g.Tf + lt : sel4(tb.t0, j) + ti * sel4(tb.dt, j);
+        const int tl = ti < 0 ? lt : -1;
+        const uint32_t nb = seq_more(tb, j, ti) ? seq_recv_bytes(p.M, rank) : 0u;
         switch (g.mode) {
           case EP_RESID:
-            ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
             break;
           case EP_SWIGLU:
-            ok = seq_tile<EP_SWIGLU, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_SWIGLU, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
             break;
           case EP_QKV:
-            ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
             break;
           default:
-            ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
             break;
         }
+        // a leftover part counts for the owner that completed its columns
+        if (leader) finished += ti >= 0 || sm.left_last ? 1u : 0u;
       }
       // this CTA's share of GEMM j is written (a barrier over the epilogue threads above)
-      if (ok && leader && nt > 0) counter_add(g.done, (unsigned int)nt);
+      if (ok && leader && finished > 0) counter_add(g.done, finished);
     }
     if (!ok && leader) {
       set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
@@ -1295,11 +1358,17 @@ bool tensor_map_3d(CUtensorMap *out, const void *ptr, int d0, int d1, int d2, in
 }
 
 void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max, int max_tiles) {
-  (void)base;
-  (void)off;
   (void)rows_max;
   (void)max_tiles;
-  w.sm_count = sm_count;  // split-K partials stay in distributed shared memory: no global scratch
+  w.sm_count = sm_count;  // split-K partials of whole tiles stay in distributed shared memory
+  // the persistent launch's leftover-tile sums and counts, per GEMM slot
+  off = (off + 255) & ~(size_t)255;
+  const size_t acc_bytes = (size_t)SEQ_MAX * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD * sizeof(float);
+  const size_t ctr_bytes = (size_t)SEQ_MAX * SEQ_LEFT_MAX * SEQ_P * sizeof(unsigned int);
+  w.lacc = base ? reinterpret_cast<float *>(base + off) : nullptr;
+  w.lctr = base ? reinterpret_cast<unsigned int *>(base + off + acc_bytes) : nullptr;
+  w.left_bytes = acc_bytes + ctr_bytes;
+  off += (w.left_bytes + 255) & ~(size_t)255;
 }
 
 bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep) {
@@ -1308,9 +1377,8 @@ bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep) {
 }
 
 cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s) {
-  (void)w;
-  (void)s;
-  return cudaSuccess;
+  if (w.lacc == nullptr) return cudaSuccess;
+  return cudaMemsetAsync(w.lacc, 0, w.left_bytes, s);
 }
 
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
@@ -1362,13 +1430,18 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
   return cudaSuccess;
 }
 
+// leftover tiles split over several clusters (DFLOW_SEQ_NO_LEFTOVER: one cluster each)
+static bool seq_left_enabled() {
+  static const bool on = getenv("DFLOW_SEQ_NO_LEFTOVER") == nullptr;
+  return on;
+}
+
 bool seq_supported(int M) {
   return M >= 1 && (M + 15) / 16 * 16 <= MAX_SPLIT_NPAD && encode_fn() != nullptr;
 }
 
 cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
                      DepChain *chain) {
-  (void)w;
   if (n < 1 || n > SEQ_MAX || !chain || !chain->dev || !seq_supported(M)) return cudaErrorInvalidValue;
   SeqParams p{};
   SeqMaps maps{};
@@ -1396,19 +1469,28 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     g.T = (q.N + BM - 1) / BM;
     g.kb = q.K / BK;
     g.mode = mode;
-    // 4-way split for every GEMM.  (A 2-way split, two groups per cluster, gives
-    // the 48-tile QKV projection one tile per group on 96 CTAs instead of a
-    // second tile on 48 of 144; measured no faster at Qwen3-8B batch 1, since a
-    // CTA's weight stream is latency bound either way.)
-    g.P = SEQ_P;
+    // leftover tiles when they divide the clusters evenly and every part keeps a k-block
+    const int lo = g.T % p.Q;
+    g.Tf = g.T;
+    g.Tl = 0;
+    g.ls = 1;
+    if (lo > 0 && lo <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
+        seq_left_enabled()) {
+      g.Tf = g.T - lo;
+      g.Tl = lo;
+      g.ls = p.Q / lo;
+      g.lacc = w.lacc + (size_t)j * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD;
+      g.lctr = w.lctr + (size_t)j * SEQ_LEFT_MAX * SEQ_P;
+    }
     g.idesc = idesc;
     g.ep = q.ep;
     g.ep.qkv.row0 = 0;
     if (!tensor_map(&maps.w[j], q.W, q.N, q.K, q.K, BM) || !tensor_map(&maps.x[j], q.X, M, q.K, q.ldx, p.npad))
       return cudaErrorInvalidValue;
   }
-  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc((unsigned)(p.g[j].P * p.g[j].T), &p.g[j].done_n);
-  const Dep d = chain->take((unsigned)(p.g[n - 1].P * p.g[n - 1].T));
+  auto done_count = [&](const SeqGemm &g) { return (unsigned)(SEQ_P * g.T); };  // each owner once per tile
+  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc(done_count(p.g[j]), &p.g[j].done_n);
+  const Dep d = chain->take(done_count(p.g[n - 1]));
   p.g[n - 1].done = d.signal;
   p.g[n - 1].done_n = chain->shadow[chain->last];
   p.dep = d;

@@ -15,11 +15,12 @@ bool tensor_map_3d(CUtensorMap *out, const void *ptr, int d0, int d1, int d2, in
 
 // Scratch of the tensor-core GEMM inside the handle's workspace.
 struct TcWorkspace {
-  float *part = nullptr;   // split-K partial tiles
-  int *counters = nullptr; // per-tile arrival counters (left at zero after every launch)
-  size_t part_elems = 0;
-  int n_counters = 0;
   int sm_count = 0;
+  // persistent launch: fp32 sums and arrival counts of tiles split over several
+  // clusters (zero between uses; tc_init zeroes them)
+  float *lacc = nullptr;
+  unsigned int *lctr = nullptr;
+  size_t left_bytes = 0;
 };
 
 // Reserve the GEMM scratch at byte offset `off` of `base` (null base: size only).
