@@ -342,7 +342,6 @@ struct LeftPart {
 __device__ __forceinline__ void red_add_v4(float *a, float x, float y, float z, float w) {
   asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(a), "f"(x), "f"(y), "f"(z), "f"(w) : "memory");
 }
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsigned int v) {
   unsigned int old;
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
@@ -362,10 +361,10 @@ __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsign
 // CW4 > 0: the split is 4-way over npad = 4 CW4 columns (each owner finishes
 // CW4 of them), known at compile time: every loop has a fixed trip count, the
 // owner of a column group is a constant, and the epilogue covers CW4 columns.
-template <int EP, typename PT, int CW4 = 0>
 // lp.acc set (CW4 > 0 only): the cluster holds one part of the tile; each owner
 // adds its columns' sum into lp.acc and only the one completing the count runs
 // their epilogue (sm.left_last = 1 in that CTA).
+template <int EP, typename PT, int CW4 = 0>
 __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P_, int npad_, int M,
                                             uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
                                             int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n,
@@ -468,7 +467,9 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
 #pragma unroll
           for (int q4 = 0; q4 < NC / 4; ++q4)
             if (c0 + 4 * q4 < s1) red_add_v4(a + 4 * q4, v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
-          fence_acq_rel_gpu();  // this thread's additions are visible before the count below
+          // the leader's count is a release at GPU scope that follows every thread's
+          // additions through the barrier (the pattern of a block-wide result
+          // published by one thread), and an acquire for the last part's reads
           epi_bar();
           if (leader) sm.left_last = atom_add_acq_rel(lp.ctr, 1u) == lp.parts - 1 ? 1 : 0;
           epi_bar();
