@@ -119,6 +119,66 @@ __device__ __forceinline__ void column_sums(Smem &sm, int sub, int lane, const f
   epi_bar();
 }
 
+// sm.col_scale[c] = rsqrt(sum_e in_ss[e][c] / d + eps) for the M columns: the
+// input rows' RMSNorm folded into the product.  All 128 epilogue threads load
+// (a column and a stride of the partials each, so the L2 loads overlap), then
+// the groups' sums are added in a fixed order.
+__device__ __forceinline__ void col_scales(const EpArgs &ep, Smem &sm, int M, int r) {
+  if (M > 64) {
+    for (int c = r; c < M; c += BM) {
+      float acc0 = 0.f, acc1 = 0.f;
+      int e = 0;
+#pragma unroll 4
+      for (; e + 1 < ep.in_ss_n; e += 2) {
+        acc0 += __ldcg(ep.in_ss + (size_t)e * ep.ld_ss + c);
+        acc1 += __ldcg(ep.in_ss + (size_t)(e + 1) * ep.ld_ss + c);
+      }
+      if (e < ep.in_ss_n) acc0 += __ldcg(ep.in_ss + (size_t)e * ep.ld_ss + c);
+      sm.col_scale[c] = rsqrtf((acc0 + acc1) * ep.in_inv_d + ep.in_eps);
+    }
+    epi_bar();
+    return;
+  }
+  const int cols = M <= 32 ? 32 : 64, groups = BM / cols;
+  const int c = r % cols, q = r / cols;
+  const float *const src = ep.in_ss + c;
+  const int n = ep.in_ss_n;
+  const size_t ld = ep.ld_ss;
+  float acc0 = 0.f, acc1 = 0.f;
+  if (c < M) {
+    int e = q;
+#pragma unroll 4
+    for (; e + groups < n; e += 2 * groups) {
+      acc0 += __ldcg(src + (size_t)e * ld);
+      acc1 += __ldcg(src + (size_t)(e + groups) * ld);
+    }
+    if (e < n) acc0 += __ldcg(src + (size_t)e * ld);
+  }
+  float *const part = &sm.xch[0][0];  // [groups][cols]
+  part[q * cols + c] = acc0 + acc1;
+  epi_bar();
+  if (r < M) {
+    float tot = 0.f;
+    for (int g = 0; g < groups; ++g) tot += part[g * cols + r];
+    sm.col_scale[r] = rsqrtf(tot * ep.in_inv_d + ep.in_eps);
+  }
+  epi_bar();
+}
+
+// token column -> position and paged-pool slot of the Q/K/V epilogue
+__device__ __forceinline__ void qkv_table(const QkvOut &o, Smem &sm, int M, int r) {
+  for (int c = r; c < M; c += BM) {
+    const int grow = o.row0 + c, pp = o.pos[grow];
+    long long base = -1;
+    if (o.bk == nullptr && o.wr[grow]) {
+      const int page = o.page_table[(size_t)(grow / o.R) * o.pages_per_seq + pp / o.page_size];
+      base = ((long long)page * 2 * o.hkv * o.page_size + pp % o.page_size) * BM;
+    }
+    sm.qkv_pos[c] = pp;
+    sm.qkv_base[c] = base;
+  }
+}
+
 // prefetch of the inputs epilogue_chunk(t, c0, nc) will need (PT: any parameter
 // block with the GEMM's N, M and ep)
 template <int EP, typename PT, int NC = 16>
@@ -638,28 +698,10 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
     const bool leader = threadIdx.x == 64;
     if (leader) dep_wait(p.dep, p.status);
     epi_bar();  // the other epilogue threads read the previous launch's outputs after the leader's wait
-    if (p.ep.in_ss) {
-      // the input rows' RMSNorm, folded into a per-column scale of the product
-      for (int c = r; c < p.M; c += BM) {
-        float acc = 0.f;
-        for (int i = 0; i < p.ep.in_ss_n; ++i) acc += __ldcg(p.ep.in_ss + (size_t)i * p.ep.ld_ss + c);
-        sm.col_scale[c] = rsqrtf(acc * p.ep.in_inv_d + p.ep.in_eps);
-      }
-      epi_bar();
-    }
+    if (p.ep.in_ss) col_scales(p.ep, sm, p.M, r);
     if constexpr (EP == EP_QKV) {
       // per token column: position, and the paged-pool slot its K/V rows go to
-      const QkvOut &o = p.ep.qkv;
-      for (int c = r; c < p.M; c += BM) {
-        const int grow = o.row0 + c, pp = o.pos[grow];
-        long long base = -1;
-        if (o.bk == nullptr && o.wr[grow]) {
-          const int page = o.page_table[(size_t)(grow / o.R) * o.pages_per_seq + pp / o.page_size];
-          base = ((long long)page * 2 * o.hkv * o.page_size + pp % o.page_size) * BM;
-        }
-        sm.qkv_pos[c] = pp;
-        sm.qkv_base[c] = base;
-      }
+      qkv_table(p.ep.qkv, sm, p.M, r);
       epi_bar();
     }
     int i = 0;
@@ -1038,29 +1080,13 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
           set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
       }
       epi_bar();
-      if (g.ep.in_ss) {
-        // the input rows' RMSNorm, folded into a per-column scale of the product
-        for (int c = r; c < p.M; c += BM) {
-          float acc = 0.f;
-          for (int e = 0; e < g.ep.in_ss_n; ++e) acc += __ldcg(g.ep.in_ss + (size_t)e * g.ep.ld_ss + c);
-          sm.col_scale[c] = rsqrtf(acc * g.ep.in_inv_d + g.ep.in_eps);
-        }
+      // positions and pool slots of the Q/K/V projection (the last GEMM, if any)
+      // come from before this launch: set up while the first GEMM streams
+      if (j == 0 && p.g[p.n - 1].mode == EP_QKV) {
+        qkv_table(p.g[p.n - 1].ep.qkv, sm, p.M, r);
         epi_bar();
       }
-      if (g.mode == EP_QKV) {
-        const QkvOut &o = g.ep.qkv;
-        for (int c = r; c < p.M; c += BM) {
-          const int grow = o.row0 + c, pp = o.pos[grow];
-          long long base = -1;
-          if (o.bk == nullptr && o.wr[grow]) {
-            const int page = o.page_table[(size_t)(grow / o.R) * o.pages_per_seq + pp / o.page_size];
-            base = ((long long)page * 2 * o.hkv * o.page_size + pp % o.page_size) * BM;
-          }
-          sm.qkv_pos[c] = pp;
-          sm.qkv_base[c] = base;
-        }
-        epi_bar();
-      }
+      if (g.ep.in_ss) col_scales(g.ep, sm, p.M, r);
       const int nt = sel4(tb.nt, j), lt = sel4(tb.lt, j);
       unsigned int finished = 0;  // tiles whose columns of this CTA are written
       for (int ti = lt >= 0 ? -1 : 0; ti < nt && ok; ++ti, ++i) {
@@ -1461,7 +1487,8 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     const SeqSpec &q = sp[j];
     const int mode = q.ep.mode;
     if (q.K % BK || q.K / BK < SEQ_P || q.N < 1 || q.ldx % 8 ||
-        (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV))
+        (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV) ||
+        (mode == EP_QKV && j != n - 1))  // its column table is built once, for the last GEMM
       return cudaErrorInvalidValue;
     SeqGemm &g = p.g[j];
     g.N = q.N;
