@@ -784,6 +784,11 @@ constexpr int SEQ_LEFT_MAX = 40;  // leftover tiles of one GEMM (fewer than the 
 struct SeqGemm {
   int N, K, M, T, kb, mode;
   int Tf, Tl, ls;
+  // the per-CTA schedule without runtime divisions: cluster q has nt_a + (q < nt_b)
+  // full tiles; x / ls and x / (SEQ_P ls) are umulhi(x, ls_mag), umulhi(x, parts_mag)
+  // (exact: every dividend here times its divisor is below 2^32)
+  int nt_a, nt_b;
+  unsigned int ls_mag, parts_mag;
   uint32_t idesc;
   EpArgs ep;
   unsigned int *done;   // completion counter: each CTA adds 1 per tile whose columns it finished
@@ -855,17 +860,19 @@ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
 #pragma unroll
   for (int j = 0; j < SEQ_MAX; ++j) {
     const bool on = j < p.n;
-    const int kb = on ? p.g[j].kb : 0, Tf = on ? p.g[j].Tf : 0, Tl = on ? p.g[j].Tl : 0, ls = on ? p.g[j].ls : 1;
+    const SeqGemm &g = p.g[j];
+    const int kb = on ? g.kb : 0;
     t.t0[j] = q;
     t.dt[j] = p.Q;
-    t.nt[j] = Tf > q ? (Tf - 1 - q) / p.Q + 1 : 0;
+    t.nt[j] = on ? g.nt_a + (q < g.nt_b ? 1 : 0) : 0;
     t.k0[j] = rr * kb / SEQ_P;
     t.k1[j] = (rr + 1) * kb / SEQ_P;
-    const bool left = q < Tl * ls;
-    const int m = (q % ls) * SEQ_P + rr, parts = SEQ_P * ls;  // this CTA's part of its leftover tile
-    t.lt[j] = left ? q / ls : -1;
-    t.lk0[j] = left ? m * kb / parts : 0;
-    t.lk1[j] = left ? (m + 1) * kb / parts : 0;
+    const bool left = on && q < g.Tl * g.ls;
+    const int lt = left ? (int)__umulhi((unsigned)q, g.ls_mag) : 0;
+    const int m = (q - lt * g.ls) * SEQ_P + rr;  // this CTA's part of its leftover tile
+    t.lt[j] = left ? lt : -1;
+    t.lk0[j] = left ? (int)__umulhi((unsigned)(m * kb), g.parts_mag) : 0;
+    t.lk1[j] = left ? (int)__umulhi((unsigned)((m + 1) * kb), g.parts_mag) : 0;
   }
   return t;
 }
@@ -903,6 +910,8 @@ __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, 
 }
 
 constexpr int SEQ_THREADS = THREADS + 32;  // warp 6: the activation producer
+// the CTA's schedule in shared memory, after the Smem block
+constexpr size_t SEQ_SMEM_TAB_OFF = (sizeof(Smem) + 15) & ~(size_t)15;
 
 // NPAD: the token columns padded to 16 (p.npad), a compile-time constant so that
 // the split-K epilogue has fixed trip counts
@@ -917,10 +926,13 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
   float *rx = reinterpret_cast<float *>(ring + (size_t)p.stages * stage_bytes);  // [SEQ_P][BM][w4] split-K receive area
   Smem &sm = *reinterpret_cast<Smem *>(reinterpret_cast<uint8_t *>(rx) + p.rx_bytes);
+  SeqTab *const stab = reinterpret_cast<SeqTab *>(reinterpret_cast<uint8_t *>(&sm) + SEQ_SMEM_TAB_OFF);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int rank = (int)cluster_rank();
 
   if (threadIdx.x == 0) {
+    // this CTA's schedule, once, for every role
+    *stab = seq_tab(p, (int)blockIdx.x);
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(&sm.full[s], 2);  // one arrival (with its byte count) from each producer
       mbar_init(&sm.empty[s], 1);
@@ -935,7 +947,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // armed for this CTA's first split-K tile before the cluster barrier below
-    const SeqTab tb = seq_tab(p, (int)blockIdx.x);
+    const SeqTab tb = *stab;
     bool any = false;
     for (int j = 0; j < tb.n; ++j) any = any || sel4(tb.nt, j) > 0 || sel4(tb.lt, j) >= 0;
     mbar_expect_tx(&sm.recv, any ? seq_recv_bytes(p.M, rank) : 0u);
@@ -959,7 +971,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     // are complete.  Each arrives on the stage's full barrier with its own bytes.
     if (lane == 0) {
       const bool wp = warp == 0;
-      const SeqTab tb = seq_tab(p, (int)blockIdx.x);
+      const SeqTab tb = *stab;
       const uint64_t pol = wp ? policy_evict_first() : policy_evict_last();
       const uint32_t bytes = wp ? (uint32_t)A_BYTES : (uint32_t)(stage_bytes - A_BYTES);
       if (wp)
@@ -1026,7 +1038,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       uint32_t ph = 0;
       bool ok = true;
       int i = 0;
-      const SeqTab tb = seq_tab(p, (int)blockIdx.x);
+      const SeqTab tb = *stab;
       const uint32_t idesc = p.g[0].idesc;  // one row count, so one instruction descriptor for all GEMMs
       for (int j = 0; j < tb.n && ok; ++j) {
         const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j), lt = sel4(tb.lt, j);
@@ -1066,7 +1078,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     const int r = sub * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
     const bool leader = threadIdx.x == 64;
-    const SeqTab tb = seq_tab(p, (int)blockIdx.x);
+    const SeqTab tb = *stab;
     bool ok = true;
     int i = 0;
     for (int j = 0; j < p.n && ok; ++j) {
@@ -1261,11 +1273,12 @@ size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
   const int stage_bytes = A_BYTES + npad * BK * 2;
   // receive area of the 4-way split: a [BM][npad / 4] fp32 slot per rank
   const size_t red_bytes = (size_t)SEQ_P * BM * (npad / SEQ_P) * 4;
-  int stages = (int)((SMEM_BUDGET - red_bytes - sizeof(Smem) - 1024) / stage_bytes);
+  const size_t tail = SEQ_SMEM_TAB_OFF + sizeof(SeqTab);  // Smem, then the schedule
+  int stages = (int)((SMEM_BUDGET - red_bytes - tail - 1024) / stage_bytes);
   if (stages > 16) stages = 16;
   *stages_out = stages;
   *rx_bytes_out = (int)red_bytes;
-  return 1024 + (size_t)stages * stage_bytes + red_bytes + sizeof(Smem);
+  return 1024 + (size_t)stages * stage_bytes + red_bytes + tail;
 }
 
 // clusters of SEQ_P persistent CTAs that are resident at once
@@ -1510,6 +1523,10 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
       g.lacc = w.lacc + (size_t)j * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD;
       g.lctr = w.lctr + (size_t)j * SEQ_LEFT_MAX * SEQ_P;
     }
+    g.nt_a = g.Tf / p.Q;
+    g.nt_b = g.Tf % p.Q;
+    g.ls_mag = g.ls > 1 ? (unsigned)((((uint64_t)1 << 32) + g.ls - 1) / g.ls) : 0u;
+    g.parts_mag = (unsigned)((((uint64_t)1 << 32) + SEQ_P * g.ls - 1) / (SEQ_P * g.ls));
     g.idesc = idesc;
     g.ep = q.ep;
     g.ep.qkv.row0 = 0;
