@@ -536,14 +536,32 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   const int *pt = a.page_table + (size_t)b * D.pages_per_seq;
   const uint64_t pol = policy_evict_first();
 
-  // warp 0: the K/V (and Q) copies that do not wait for a free stage start right
-  // after the dependency wait, before the CTA-wide barrier
-  int pg = 0, n_pre = 0, nk = 0;
+  // Before the dependency wait (so that a CTA started early does its set-up and
+  // first copies while the previous launch finishes): the key count, and the
+  // K/V pages that hold only keys from before this round's block.  Those were
+  // written by kernels that finished before the small kernel that heads this
+  // chain of launches began (each small kernel waits for its predecessor's
+  // completion before its dependents may start), as were the key counts; the
+  // page table is the caller's.  Q and the pages with the block's own rows,
+  // written by the projection just before, are read after the wait.
+  int pg = 0, n_pre = 0, n_early = 0;
+  const int nk = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;
+  auto issue_page = [&](int it, int page) {  // warp 0, lane 0: page tile `page` into stage it
+    uint8_t *kt = ring + (size_t)it * 2 * TILE, *vt = kt + TILE;
+    const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;
+    mbar_expect_tx(&sm.kv_full[it], 2 * TILE);
+    tma_load_2d(kt, &tm, 0, rk, &sm.kv_full[it], pol);
+    tma_load_2d(kt + 8192, &tm, 64, rk, &sm.kv_full[it], pol);
+    tma_load_2d(vt, &tm, 0, rv, &sm.kv_full[it], pol);
+    tma_load_2d(vt + 8192, &tm, 64, rv, &sm.kv_full[it], pol);
+  };
   if (warp == 0) {
-    // page ids of this split's first 32 pages: the page table is the caller's
-    // and does not change during a call
+    // page ids of this split's first 32 pages
     const int t = split + T5_SPLITS * lane;
     pg = t < D.pages_per_seq ? __ldg(pt + t) : 0;
+    const int n_old = a.causal ? nk - R : nk;  // pool keys older than this round's block
+    n_pre = min(t5_pool_tiles((nk + 63) / 64, split), T5_STAGES);
+    while (n_early < n_pre && (split + T5_SPLITS * n_early + 1) * 64 <= n_old) ++n_early;
     if (lane == 0) {
       prefetch_tensormap(&tm);
       if (q_tma) prefetch_tensormap(&tq);
@@ -560,49 +578,23 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
       mbar_init(&sm.q_full, q_tma ? 1 : 4);
       mbar_init(&sm.drain, 1);
       asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-      dep_wait(a.dep, status);
-      nk = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;  // consumed after the first copies are issued
-      if (a.dep.wait) fence_proxy_async_global();  // Q and K/V rows just written by the projection, read by TMA
-      if (q_tma) {
-        const uint32_t qbytes = (uint32_t)(R * G * 128);
-        mbar_expect_tx(&sm.q_full, 2 * qbytes);
-        tma_load_3d(qs, &tq, 0, kvh * G, b * R, &sm.q_full);
-        tma_load_3d(qs + T5_ROWS * 128, &tq, 64, kvh * G, b * R, &sm.q_full);
-      }
+      sm.n_keys = nk;
     }
-    __syncwarp();  // the other lanes read the previous launches' outputs after lane 0's wait
-    if constexpr (BLOCK) {
-      // drafter: the block's own tile follows the pool pages, so the key count
-      // decides the first fills
-      nk = __shfl_sync(0xffffffffu, nk, 0);
-      n_pre = min(t5_pool_tiles((nk + 63) / 64, split), T5_STAGES);
-    } else {
-      // the split's first pages go out before the key count is known: a page
-      // past the context is loaded but never consumed (its copy is still
-      // drained), a page id past the pool reads as fill
-      n_pre = min(T5_STAGES, (D.pages_per_seq - split + T5_SPLITS - 1) / T5_SPLITS);
-    }
-    for (int it = 0; it < n_pre; ++it) {
+    for (int it = 0; it < n_early; ++it) {
       const int page = __shfl_sync(0xffffffffu, pg, it);
-      if (lane == 0) {
-        uint8_t *kt = ring + (size_t)it * 2 * TILE, *vt = kt + TILE;
-        const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;
-        mbar_expect_tx(&sm.kv_full[it], 2 * TILE);
-        tma_load_2d(kt, &tm, 0, rk, &sm.kv_full[it], pol);
-        tma_load_2d(kt + 8192, &tm, 64, rk, &sm.kv_full[it], pol);
-        tma_load_2d(vt, &tm, 0, rv, &sm.kv_full[it], pol);
-        tma_load_2d(vt + 8192, &tm, 64, rv, &sm.kv_full[it], pol);
-      }
+      if (lane == 0) issue_page(it, page);
     }
-    if (lane == 0) sm.n_keys = nk;
   } else if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
                  "r"(T5_TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+  // without the Q map every softmax thread loads its own query row: then every
+  // thread is ordered after the wait by the barrier below
+  if (!q_tma && threadIdx.x == 0) dep_wait(a.dep, status);
   tc_fence_before();
-  __syncthreads();  // barriers, TMEM and the key count are in place; thread 0's wait orders every later read
+  __syncthreads();  // barriers, TMEM and the key count are in place
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
   const uint32_t t_o = tmem, t_s = tmem + 128;
@@ -610,6 +602,25 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   const int n_tiles = (n_keys + 63) / 64;
   const int Tp = t5_pool_tiles(n_tiles, split);
   const int T = Tp + ((BLOCK && split == T5_SPLITS - 1) ? 1 : 0);
+
+  if (warp == 0) {
+    // the projection's outputs: Q, then the first pages that hold block rows
+    if (lane == 0) {
+      if (q_tma) dep_wait(a.dep, status);
+      if (a.dep.wait) fence_proxy_async_global();  // rows just written by the projection, read by TMA
+      if (q_tma) {
+        const uint32_t qbytes = (uint32_t)(R * G * 128);
+        mbar_expect_tx(&sm.q_full, 2 * qbytes);
+        tma_load_3d(qs, &tq, 0, kvh * G, b * R, &sm.q_full);
+        tma_load_3d(qs + T5_ROWS * 128, &tq, 64, kvh * G, b * R, &sm.q_full);
+      }
+    }
+    for (int it = n_early; it < n_pre; ++it) {
+      const int page = __shfl_sync(0xffffffffu, pg, it);
+      if (lane == 0) issue_page(it, page);
+    }
+    __syncwarp();  // the other lanes read the projection's outputs (block rows) after lane 0's wait
+  }
 
   if (warp == 0) {
     // ---------------- producer: the remaining K/V pages ----------------
