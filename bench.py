@@ -36,7 +36,11 @@ def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=56)
-    p.add_argument("--warmup", type=int, default=4)
+    # a fresh process runs its first ~80 rounds up to 15 % slower (a GPU-side
+    # warm-up of this workload: clocks and power were steady, and neither a
+    # matmul nor a copy burn beforehand removed it); 100 rounds reach the
+    # steady state
+    p.add_argument("--warmup", type=int, default=100)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(synth.CONFIGS))
     p.add_argument("--relay", type=int, default=1, help="0 runs the DFlash baseline (no carry)")
@@ -392,6 +396,26 @@ def main():
         e2e = {"value": round(e2e_value, 2), "unit": "tokens/s",
                "h2d_bytes_per_step": 4 * cfg.batch, "d2h_bytes_per_step": 4 * cfg.batch * (1 + cfg.rows)}
 
+    # ---- per-step split: the round's four calls one at a time, events between them
+    restore()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    for k in range(K):
+        e = evs[k]
+        e[0].record(stream)
+        blk = eng.draft_block(st)
+        e[1].record(stream)
+        g_t, feats, _ = eng.verify_block(st, blk)
+        e[2].record(stream)
+        a_k, _ = eng.accept_commit(st, blk, g_t, forced_dev[Wm + k])
+        e[3].record(stream)
+        eng.carry_hidden(st, blk, feats, a_k)
+        e[4].record(stream)
+    torch.cuda.synchronize()
+    st_code = eng.read_status(st)
+    assert st_code == 0, f"device status {st_code} set during the per-step leg"
+    step_split = {name: round(float(np.median([evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(K)])), 4)
+                  for i, name in enumerate(("draft", "verify", "accept", "carry"))}
+
     # ---- profiled leg: per-launch events around the GEMMs (the dominant kernel)
     restore()
     eng.profile(True)
@@ -426,6 +450,7 @@ def main():
         "round_roofline": {"bound": "hbm", "alg_bytes": rb["total"], "achieved": round(round_gbs, 1), "peak": hbm,
                            "frac": round(round_gbs / hbm, 4), "unit": "GB/s", "peak_source": peak_src},
         "phase_ms": {"gemm": round(g["ms"] / K, 4), "attention": round(prof["attn"]["ms"] / K, 4)},
+        "step_split_ms": step_split,
         "gpu_launches": int(launches),
         "e2e": e2e,
         "clocks": clocks.summary(),

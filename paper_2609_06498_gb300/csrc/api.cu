@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cstdio>
 #include <new>
 #include <vector>
 
@@ -447,10 +448,16 @@ struct dflow_handle {
 
 namespace {
 
-#define CK(expr)                                     \
-  do {                                               \
-    cudaError_t e_ = (expr);                         \
-    if (e_ != cudaSuccess) return DFLOW_ERR_CUDA;    \
+// a failed CUDA call; with DFLOW_DEBUG set, the call and the error go to stderr
+dflow_status cuda_failed(const char *what, cudaError_t e) {
+  static const bool dbg = getenv("DFLOW_DEBUG") != nullptr;
+  if (dbg) fprintf(stderr, "dflow: %s: %s\n", what, cudaGetErrorString(e));
+  return DFLOW_ERR_CUDA;
+}
+#define CK(expr)                                           \
+  do {                                                     \
+    cudaError_t e_ = (expr);                               \
+    if (e_ != cudaSuccess) return cuda_failed(#expr, e_);  \
   } while (0)
 
 // a launch outside the counting chain: the next counting launch waits for its grid
