@@ -36,11 +36,7 @@ def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=56)
-    # a fresh process runs its first ~80 rounds up to 15 % slower (a GPU-side
-    # warm-up of this workload: clocks and power were steady, and neither a
-    # matmul nor a copy burn beforehand removed it); 100 rounds reach the
-    # steady state
-    p.add_argument("--warmup", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=8)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(synth.CONFIGS))
     p.add_argument("--relay", type=int, default=1, help="0 runs the DFlash baseline (no carry)")

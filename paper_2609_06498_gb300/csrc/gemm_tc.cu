@@ -392,16 +392,16 @@ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
   return s1 > s0 ? (uint32_t)((P - 1) * BM * ((s1 - s0 + 3) / 4) * 16) : 0u;
 }
 
-// A cluster's part of a tile that several clusters share: the fp32 sums of the
-// tile [BM][npad], the arrival count of this CTA's columns, and the parts.
+// A cluster's part of a tile that several clusters share: the tile's part slots
+// ([parts][BM][npad] fp32, slot `part` this cluster's), the arrival count of
+// this CTA's columns, and the number of parts.
 struct LeftPart {
   float *acc = nullptr;
   unsigned int *ctr = nullptr;
   unsigned int parts = 0;
+  int part = 0;
+  bool first = false;  // the group's first part: counts the tile for an owner without columns
 };
-__device__ __forceinline__ void red_add_v4(float *a, float x, float y, float z, float w) {
-  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(a), "f"(x), "f"(y), "f"(z), "f"(w) : "memory");
-}
 __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsigned int v) {
   unsigned int old;
   asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
@@ -422,8 +422,9 @@ __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsign
 // CW4 of them), known at compile time: every loop has a fixed trip count, the
 // owner of a column group is a constant, and the epilogue covers CW4 columns.
 // lp.acc set (CW4 > 0 only): the cluster holds one part of the tile; each owner
-// adds its columns' sum into lp.acc and only the one completing the count runs
-// their epilogue (sm.left_last = 1 in that CTA).
+// stores its columns' sum in its part's slot, and only the one completing the
+// count adds the parts (in part order, so the result does not depend on the
+// arrival order) and runs their epilogue (sm.left_last = 1 in that CTA).
 template <int EP, typename PT, int CW4 = 0>
 __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, int P_, int npad_, int M,
                                             uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
@@ -479,6 +480,8 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
   __syncwarp();
   epi_bar();
   const bool ok = sm.flag != 0;
+  // a shared tile counts once per column owner: for an owner without columns, in its first part
+  if (leader) sm.left_last = (lp.acc != nullptr && s0 >= s1 && lp.first) ? 1 : 0;
   // re-arm recv for the next tile, then let the senders push again; done right
   // after the last read of the receive area, before the epilogue's global
   // stores (which a release arrive issued after them would wait for)
@@ -522,11 +525,14 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
       if (c0 > s0) epilogue_prefetch<EP, PT, NC>(g, sm, t, r, c0, min(NC, s1 - c0), pre);
       if constexpr (CW4 > 0) {
         if (lp.acc != nullptr) {
-          // one chunk (CW4 <= 16): this cluster's part of the columns into the tile's sums
+          // one chunk (CW4 <= 16): this cluster's part of the columns into its slot
+          const size_t slot = (size_t)BM * npad;
           float *const a = lp.acc + (size_t)r * npad + c0;
 #pragma unroll
           for (int q4 = 0; q4 < NC / 4; ++q4)
-            if (c0 + 4 * q4 < s1) red_add_v4(a + 4 * q4, v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]);
+            if (c0 + 4 * q4 < s1)
+              __stcg(reinterpret_cast<float4 *>(a + lp.part * slot + 4 * q4),
+                     make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
           // the leader's count is a release at GPU scope that follows every thread's
           // additions through the barrier (the pattern of a block-wide result
           // published by one thread), and an acquire for the last part's reads
@@ -534,13 +540,19 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
           if (leader) sm.left_last = atom_add_acq_rel(lp.ctr, 1u) == lp.parts - 1 ? 1 : 0;
           epi_bar();
           if (!sm.left_last) continue;
-          // every part is in (the leader's acquire, ordered before these reads by the barrier):
-          // the sums, leaving zeros for the next use
+          // every part is in (the leader's acquire, ordered before these reads by the
+          // barrier): their sum in part order; the count is left at zero
 #pragma unroll
           for (int q4 = 0; q4 < NC / 4; ++q4) {
             if (c0 + 4 * q4 >= s1) break;
-            const float4 x = __ldcg(reinterpret_cast<const float4 *>(a + 4 * q4));
-            __stcg(reinterpret_cast<float4 *>(a + 4 * q4), make_float4(0.f, 0.f, 0.f, 0.f));
+            float4 x = __ldcg(reinterpret_cast<const float4 *>(a + 4 * q4));
+            for (int pp = 1; pp < (int)lp.parts; ++pp) {
+              const float4 y = __ldcg(reinterpret_cast<const float4 *>(a + pp * slot + 4 * q4));
+              x.x += y.x;
+              x.y += y.y;
+              x.z += y.z;
+              x.w += y.w;
+            }
             v[4 * q4] = x.x;
             v[4 * q4 + 1] = x.y;
             v[4 * q4 + 2] = x.z;
@@ -771,16 +783,17 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
 // ===========================================================================
 constexpr int SEQ_MAX = 4;  // GEMMs per launch
 constexpr int SEQ_P = 4;    // cluster size = split-K ways of a tile inside a cluster
-constexpr int SEQ_LEFT_MAX = 40;  // leftover tiles of one GEMM (fewer than the clusters, at most 38)
+constexpr int SEQ_LEFT_MAX = 40;  // leftover tiles of one GEMM and part slots (one per cluster; at most 38)
 
 // Tiles 0 .. Tf-1 go to the Q clusters round robin (cluster q: q, q + Q, ...),
 // each split 4 ways over the cluster's CTAs and reduced in shared memory.  The
 // Tl = T - Tf leftover tiles (T mod Q of them, when Q is a multiple) are each
 // split over ls = Q / Tl clusters, 4 ls ways: every CTA then streams the same
 // number of weight k-blocks.  A cluster reduces its part of a leftover tile in
-// shared memory like any tile; each column owner then adds its columns in fp32
-// into lacc (L2), and the owner whose addition completes the count of its
-// columns runs their epilogue and leaves lacc and the count at zero again.
+// shared memory like any tile; each column owner then stores its columns in
+// its cluster's fp32 slot of lacc (L2), and the owner whose arrival completes
+// the count of its columns adds the slots in part order, runs their epilogue
+// and leaves the count at zero again.
 struct SeqGemm {
   int N, K, M, T, kb, mode;
   int Tf, Tl, ls;
@@ -793,7 +806,7 @@ struct SeqGemm {
   EpArgs ep;
   unsigned int *done;   // completion counter: each CTA adds 1 per tile whose columns it finished
   unsigned int done_n;  // its value once every tile of this GEMM is finished
-  float *lacc;          // [Tl][BM][npad] leftover sums (zero between uses)
+  float *lacc;          // [Q][BM][npad] leftover part slots, one per cluster
   unsigned int *lctr;   // [Tl][SEQ_P] leftover contributions per column owner (zero between uses)
 };
 struct SeqMaps {
@@ -848,6 +861,7 @@ __device__ __forceinline__ const CUtensorMap *seq_xmap(const SeqMaps &m, int j) 
 struct SeqTab {
   int n, nt[SEQ_MAX], t0[SEQ_MAX], dt[SEQ_MAX], k0[SEQ_MAX], k1[SEQ_MAX];
   int lt[SEQ_MAX], lk0[SEQ_MAX], lk1[SEQ_MAX];  // leftover tile (index among the leftovers, or -1) and k range
+  int lpart[SEQ_MAX];                           // the cluster's part index in its leftover tile
 };
 __device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
   return j == 0 ? a[0] : j == 1 ? a[1] : j == 2 ? a[2] : a[3];
@@ -871,6 +885,7 @@ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
     const int lt = left ? (int)__umulhi((unsigned)q, g.ls_mag) : 0;
     const int m = (q - lt * g.ls) * SEQ_P + rr;  // this CTA's part of its leftover tile
     t.lt[j] = left ? lt : -1;
+    t.lpart[j] = left ? q - lt * g.ls : 0;
     t.lk0[j] = left ? (int)__umulhi((unsigned)(m * kb), g.parts_mag) : 0;
     t.lk1[j] = left ? (int)__umulhi((unsigned)((m + 1) * kb), g.parts_mag) : 0;
   }
@@ -895,13 +910,17 @@ __device__ __forceinline__ bool seq_more(const SeqTab &tb, int j, int ti) {
 // lt >= 0: t is leftover tile lt, the cluster holds one part of it.
 template <int EP, int NPAD>
 __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, uint32_t lane_addr, int i, int t, int lt,
-                                         int r, int sub, int lane, int rank, bool leader, uint32_t next_bytes) {
+                                         int part, int r, int sub, int lane, int rank, bool leader,
+                                         uint32_t next_bytes) {
   static_assert(SEQ_P == 4, "the compile-time split of splitk_tile is 4-way");
   LeftPart lp;
   if (lt >= 0) {
-    lp.acc = g.lacc + (size_t)lt * BM * NPAD;
+    // slots of clusters lt ls .. lt ls + ls - 1 (one per cluster of the GEMM)
+    lp.acc = g.lacc + (size_t)lt * g.ls * BM * NPAD;
     lp.ctr = g.lctr + lt * SEQ_P + rank;
     lp.parts = (unsigned int)g.ls;
+    lp.part = part;
+    lp.first = part == 0;
   }
   const bool ok = splitk_tile<EP, SeqGemm, NPAD / 4>(g, sm, rx, SEQ_P, NPAD, g.M, lane_addr, i, t, r, sub, lane, rank, 0,
                                                      leader, next_bytes, 1u, lp);
@@ -945,6 +964,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     mbar_init(&sm.rfree, SEQ_P - 1);
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
+    sm.left_last = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     // armed for this CTA's first split-K tile before the cluster barrier below
     const SeqTab tb = *stab;
@@ -1104,26 +1124,31 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       for (int ti = lt >= 0 ? -1 : 0; ti < nt && ok; ++ti, ++i) {
         const int t = ti < 0 ? g.Tf + lt : sel4(tb.t0, j) + ti * sel4(tb.dt, j);
         const int tl = ti < 0 ? lt : -1;
+        const int fp = ti < 0 ? sel4(tb.lpart, j) : 0;  // the cluster's part of its leftover tile
         const uint32_t nb = seq_more(tb, j, ti) ? seq_recv_bytes(p.M, rank) : 0u;
         switch (g.mode) {
           case EP_RESID:
-            ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
           case EP_SWIGLU:
-            ok = seq_tile<EP_SWIGLU, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_SWIGLU, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
           case EP_QKV:
-            ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
           default:
-            ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, tl, r, sub, lane, rank, leader, nb);
+            ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
         }
         // a leftover part counts for the owner that completed its columns
         if (leader) finished += ti >= 0 || sm.left_last ? 1u : 0u;
       }
-      // this CTA's share of GEMM j is written (a barrier over the epilogue threads above)
-      if (ok && leader && finished > 0) counter_add(g.done, finished);
+      // this CTA's share of GEMM j is written (a barrier over the epilogue threads above);
+      // a count past the GEMM's target would release a later wait on this counter early
+      if (ok && leader && finished > 0) {
+        const unsigned int old = atom_add_acq_rel(g.done, finished);
+        if ((int)(old + finished - g.done_n) > 0) set_status(p.status, DFLOW_ERR_BAD_STATE);
+      }
     }
     if (!ok && leader) {
       set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
@@ -1515,7 +1540,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     g.Tf = g.T;
     g.Tl = 0;
     g.ls = 1;
-    if (lo > 0 && lo <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
+    if (lo > 0 && p.Q <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
         seq_left_enabled()) {
       g.Tf = g.T - lo;
       g.Tl = lo;

@@ -139,6 +139,39 @@ def test_full_depth_8b_round_invariants():
     assert eng.read_status(st) == 0
 
 
+def test_full_depth_8b_many_rounds_stay_clean_and_deterministic():
+    """120 rounds of the benchmark workload through the round call: every
+    bounded wait holds and no completion count passes its target (either sets
+    the device status); the sequence grows by the forced acceptance.  A second
+    engine state replaying the same rounds gives bit-identical target tokens and
+    features (the split-K sums, across clusters too, have a fixed order)."""
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = synth.QWEN3_8B
+    rounds = 120
+    eng = Engine(cfg, random_weights(cfg, seed=0), max_batch=1,
+                 max_ctx=cfg.replace(new_tokens=rounds * cfg.rows).max_ctx())
+    sched = synth.forced_schedule(cfg, rounds)
+    runs = []
+    for _ in range(2):
+        st = eng.new_state(1, page_seed=3)
+        eng.prefill(st, synth.prompts(cfg))
+        n0 = int(st.seq_len[0])
+        toks = []
+        for r in range(rounds):
+            acc, comm = eng.round(st, torch.as_tensor(sched[r]).cuda())
+            toks.append(to_np(comm)[0].copy())
+        assert eng.read_status(st) == 0
+        assert int(st.seq_len[0]) == n0 + int((sched[:, 0] + 1).sum())
+        blk = eng.draft_block(st)
+        g, feats, _ = eng.verify_block(st, blk)
+        runs.append((np.array(toks), to_np(blk), to_np(g), to_np(feats)))
+        assert eng.read_status(st) == 0
+        del st
+    for x, y in zip(runs[0], runs[1]):
+        assert np.array_equal(x, y)
+
+
 def test_batch16_long_context_rounds_stay_clean():
     """Forty rounds of the batch-16, 8K-context shape (2 + 1 layers, full widths):
     no bounded device wait may expire, and every sequence grows by exactly its
