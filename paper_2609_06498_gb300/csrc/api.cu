@@ -572,6 +572,14 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
   const double es = h->esz;
   ProfScope ps(h, k.s, DFLOW_PROF_GEMM, es * N * K + es * M * K + ep_out_bytes(ep, M, N, h->esz), 2.0 * M * N * K);
   ++h->n_launch;
+  // few rows: the persistent kernel, one GEMM (all 36 clusters, balanced tiles)
+  static const bool single_tc = getenv("DFLOW_GEMM_TC_SINGLE") != nullptr;
+  const bool seq_mode = ep.mode == EP_STORE_F32 || ep.mode == EP_RESID || ep.mode == EP_SWIGLU || ep.mode == EP_QKV;
+  if (h->use_tc && !single_tc && seq_mode && h->dep.dev != nullptr && K % 64 == 0 && K / 64 >= 4 &&
+      ldx % 8 == 0 && seq_supported(M)) {
+    const SeqSpec sp{W, N, K, X, ldx, ep};
+    return gemm_seq(h->tcw, 1, &sp, M, k.status_w, k.s, &h->dep);
+  }
   if (h->use_tc && tc_supports(N, K, M, ldx, ep))
     return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
   h->dep.brk();
