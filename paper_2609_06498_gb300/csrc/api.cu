@@ -855,6 +855,27 @@ cudaError_t ctx_append(const Call &k, const Dims &D, int rows, const dflow_state
   dflow_handle *h = k.h;
   cudaError_t e;
   const size_t qoff = (size_t)D.hq * D.hd * D.d;  // K and V rows follow the Q rows of w_qkv
+  const int nkv = 2 * D.hkv * D.hd;
+  if (h->fused && h->dep.dev != nullptr && seq_supported(rows) && D.d % 64 == 0 && D.d / 64 >= 4) {
+    // the draft layers' projections are independent: up to four per persistent launch
+    for (int l0 = 0; l0 < h->cfg.draft_layers; l0 += 4) {
+      SeqSpec sp[4];
+      int n = 0;
+      double bytes = 0.0, flops = 0.0;
+      for (int l = l0; l < std::min(l0 + 4, h->cfg.draft_layers); ++l) {
+        const dflow_layer_weights &L = h->dl[l];
+        T *pool_l = static_cast<T *>(st->draft_kv) + (size_t)l * pool_layer_elems(D);
+        sp[n++] = SeqSpec{static_cast<const T *>(L.w_qkv) + qoff, nkv, D.d, feats, D.d,
+                          qkv_ep(h, D, 0, nullptr, L.k_norm, h->pos2, h->wr2, pool_l, st->page_table, false)};
+        bytes += (double)h->esz * nkv * D.d + (double)h->esz * rows * D.d;
+        flops += 2.0 * rows * nkv * D.d;
+      }
+      ProfScope ps(h, k.s, DFLOW_PROF_GEMM, bytes, flops);
+      ++h->n_launch;
+      if ((e = gemm_seq(h->tcw, n, sp, rows, k.status_w, k.s, &h->dep, true))) return e;
+    }
+    return cudaSuccess;
+  }
   for (int l = 0; l < h->cfg.draft_layers; ++l) {
     const dflow_layer_weights &L = h->dl[l];
     const T *wkv = static_cast<const T *>(L.w_qkv) + qoff;

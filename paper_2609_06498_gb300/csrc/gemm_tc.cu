@@ -814,6 +814,7 @@ struct SeqMaps {
 };
 struct SeqParams {
   int n, M, npad, Q, stages, tmem_cols, rx_bytes;
+  int independent;  // 1: no GEMM reads another's output; they share the launch's completion counter
   int *status;
   Dep dep;  // the previous launch: inputs of the first GEMM
   SeqGemm g[SEQ_MAX];
@@ -998,20 +999,22 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         for (int j = 0; j < tb.n; ++j) prefetch_tensormap(seq_wmap(maps, j));
       int stage = 0, u = 0;
       uint32_t ph = 0;
-      bool ok = true;
+      bool ok = true, dep_done = false;
       for (int j = 0; j < tb.n && ok; ++j) {
         const int nt = sel4(tb.nt, j), k0 = sel4(tb.k0, j), k1 = sel4(tb.k1, j), lt = sel4(tb.lt, j);
         if (nt == 0 && lt < 0) continue;
         const CUtensorMap *map = wp ? seq_wmap(maps, j) : seq_xmap(maps, j);
         if (!wp) {
           // GEMM j reads what GEMM j - 1 (or the previous launch) wrote
-          if (j == 0) {
-            dep_wait(p.dep, p.status);
+          if (j == 0 || p.independent) {
+            // the launch's inputs: once, before this producer's first copy
+            if (!dep_done) dep_wait(p.dep, p.status);
+            dep_done = true;
           } else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n)) {
             ok = false;
             break;
           }
-          if (j > 0 || p.dep.wait) fence_proxy_async_global();
+          if ((j > 0 && !p.independent) || p.dep.wait) fence_proxy_async_global();
           prefetch_tensormap(map);
         }
         // the leftover part first, then the full tiles
@@ -1108,7 +1111,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       if (leader) {
         if (j == 0)
           dep_wait(p.dep, p.status);
-        else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n))
+        else if (!p.independent && !counter_wait(p.g[j - 1].done, p.g[j - 1].done_n))
           set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
       }
       epi_bar();
@@ -1505,12 +1508,20 @@ bool seq_supported(int M) {
   return M >= 1 && (M + 15) / 16 * 16 <= MAX_SPLIT_NPAD && encode_fn() != nullptr;
 }
 
+// two Q/K/V epilogues build the same column table (positions and pool slots)
+static bool same_qkv_table(const QkvOut &a, const QkvOut &b) {
+  return a.pos == b.pos && a.wr == b.wr && a.page_table == b.page_table && a.R == b.R &&
+         a.pages_per_seq == b.pages_per_seq && a.page_size == b.page_size && a.hkv == b.hkv &&
+         (a.bk == nullptr) == (b.bk == nullptr);
+}
+
 cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
-                     DepChain *chain) {
+                     DepChain *chain, bool independent) {
   if (n < 1 || n > SEQ_MAX || !chain || !chain->dev || !seq_supported(M)) return cudaErrorInvalidValue;
   SeqParams p{};
   SeqMaps maps{};
   p.n = n;
+  p.independent = independent ? 1 : 0;
   p.M = M;
   p.npad = (M + 15) / 16 * 16;
   p.status = status;
@@ -1526,7 +1537,9 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     const int mode = q.ep.mode;
     if (q.K % BK || q.K / BK < SEQ_P || q.N < 1 || q.ldx % 8 ||
         (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV) ||
-        (mode == EP_QKV && j != n - 1))  // its column table is built once, for the last GEMM
+        // the Q/K/V column table is built once, from the last GEMM
+        (mode == EP_QKV && j != n - 1 &&
+         !(independent && sp[n - 1].ep.mode == EP_QKV && same_qkv_table(q.ep.qkv, sp[n - 1].ep.qkv))))
       return cudaErrorInvalidValue;
     SeqGemm &g = p.g[j];
     g.N = q.N;
@@ -1559,12 +1572,25 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
       return cudaErrorInvalidValue;
   }
   auto done_count = [&](const SeqGemm &g) { return (unsigned)(SEQ_P * g.T); };  // each owner once per tile
-  for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc(done_count(p.g[j]), &p.g[j].done_n);
-  const Dep d = chain->take(done_count(p.g[n - 1]));
-  p.g[n - 1].done = d.signal;
-  p.g[n - 1].done_n = chain->shadow[chain->last];
-  p.dep = d;
-  p.dep.signal = nullptr;
+  if (independent) {
+    // no GEMM waits for another: every GEMM counts into the launch's counter
+    unsigned total = 0;
+    for (int j = 0; j < n; ++j) total += done_count(p.g[j]);
+    const Dep d = chain->take(total);
+    for (int j = 0; j < n; ++j) {
+      p.g[j].done = d.signal;
+      p.g[j].done_n = chain->shadow[chain->last];
+    }
+    p.dep = d;
+    p.dep.signal = nullptr;
+  } else {
+    for (int j = 0; j + 1 < n; ++j) p.g[j].done = chain->alloc(done_count(p.g[j]), &p.g[j].done_n);
+    const Dep d = chain->take(done_count(p.g[n - 1]));
+    p.g[n - 1].done = d.signal;
+    p.g[n - 1].done_n = chain->shadow[chain->last];
+    p.dep = d;
+    p.dep.signal = nullptr;
+  }
 
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.Q * SEQ_P);

@@ -49,8 +49,11 @@ struct SeqSpec {
 bool seq_supported(int M);
 // The GEMMs of `sp` in order, in one launch: GEMM j's activations are read once
 // every tile of GEMM j - 1 is finished; the first waits for the previous launch
-// in `chain` (required), the next launch waits for the last GEMM.
+// in `chain` (required), the next launch waits for the last GEMM.  independent:
+// no GEMM reads another's output (all wait only for the previous launch; the next
+// launch waits for all of them); Q/K/V epilogues may then appear more than once
+// if they share their column table.
 cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
-                     DepChain *chain);
+                     DepChain *chain, bool independent = false);
 
 }  // namespace dflow
