@@ -574,7 +574,8 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
   ++h->n_launch;
   // few rows: the persistent kernel, one GEMM (all 36 clusters, balanced tiles)
   static const bool single_tc = getenv("DFLOW_GEMM_TC_SINGLE") != nullptr;
-  const bool seq_mode = ep.mode == EP_STORE_F32 || ep.mode == EP_RESID || ep.mode == EP_SWIGLU || ep.mode == EP_QKV;
+  const bool seq_mode = ep.mode == EP_STORE_F32 || ep.mode == EP_RESID || ep.mode == EP_SWIGLU ||
+                        ep.mode == EP_QKV || ep.mode == EP_SILU;
   if (h->use_tc && !single_tc && seq_mode && h->dep.dev != nullptr && K % 64 == 0 && K / 64 >= 4 &&
       ldx % 8 == 0 && seq_supported(M)) {
     const SeqSpec sp{W, N, K, X, ldx, ep};
@@ -912,8 +913,20 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
     KL(klaunch(k_relay_u<T>, batch * B, 256, 0, k.s, (const T *)h->w.embed, st->boundary, (const T *)st->carry,
                                              (T *)h->relay_u, D.d, B, D.vocab, k.status));
     CK(cudaGetLastError());
-    CK(gemm(k, h->w.relay_w1, D.d, 3 * D.d, h->relay_u, batch * B, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)));
-    CK(gemm(k, h->w.relay_w2, 2 * D.d, D.d, h->relay_h, batch * B, D.d, ep_f32(h->gf32, 2 * D.d)));
+    const int rr = batch * B;
+    if (h->use_tc && h->dep.dev != nullptr && seq_supported(rr) && D.d % 64 == 0) {
+      // both relay GEMMs in one persistent launch (the second reads the first's SiLU output)
+      const SeqSpec sp[2] = {{h->w.relay_w1, D.d, 3 * D.d, h->relay_u, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)},
+                             {h->w.relay_w2, 2 * D.d, D.d, h->relay_h, D.d, ep_f32(h->gf32, 2 * D.d)}};
+      ProfScope ps(h, k.s, DFLOW_PROF_GEMM,
+                   (double)h->esz * (3.0 * D.d * D.d + 2.0 * D.d * D.d) + (double)h->esz * rr * 4.0 * D.d,
+                   2.0 * rr * 5.0 * D.d * D.d);
+      ++h->n_launch;
+      CK(gemm_seq(h->tcw, 2, sp, rr, k.status_w, k.s, &h->dep));
+    } else {
+      CK(gemm(k, h->w.relay_w1, D.d, 3 * D.d, h->relay_u, rr, 3 * D.d, ep_t(EP_SILU, h->relay_h, D.d)));
+      CK(gemm(k, h->w.relay_w2, 2 * D.d, D.d, h->relay_h, rr, D.d, ep_f32(h->gf32, 2 * D.d)));
+    }
   }
   KL(klaunch(k_draft_input<T>, rows, 256, 0, k.s, (const T *)h->w.embed, h->w.e_mask, st->tokens, st->seq_len,
                                           h->cfg.max_ctx, (const T *)st->carry, st->n_carry, h->gf32,

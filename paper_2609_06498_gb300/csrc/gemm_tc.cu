@@ -1139,6 +1139,9 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
           case EP_QKV:
             ok = seq_tile<EP_QKV, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
+          case EP_SILU:
+            ok = seq_tile<EP_SILU, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
+            break;
           default:
             ok = seq_tile<EP_STORE_F32, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
             break;
@@ -1536,7 +1539,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     const SeqSpec &q = sp[j];
     const int mode = q.ep.mode;
     if (q.K % BK || q.K / BK < SEQ_P || q.N < 1 || q.ldx % 8 ||
-        (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV) ||
+        (mode != EP_STORE_F32 && mode != EP_RESID && mode != EP_SWIGLU && mode != EP_QKV && mode != EP_SILU) ||
         // the Q/K/V column table is built once, from the last GEMM
         (mode == EP_QKV && j != n - 1 &&
          !(independent && sp[n - 1].ep.mode == EP_QKV && same_qkv_table(q.ep.qkv, sp[n - 1].ep.qkv))))
