@@ -820,16 +820,19 @@ struct SeqParams {
   SeqGemm g[SEQ_MAX];
 };
 
-__device__ __forceinline__ bool counter_reached(const unsigned int *c, unsigned int n) {
-  unsigned int v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(c) : "memory");
-  return (int)(v - n) >= 0;
-}
-// bounded wait on a completion counter (acquire); false on expiry
-__device__ __forceinline__ bool counter_wait(const unsigned int *c, unsigned int n) {
+// bounded wait on a completion counter (acquire); false on expiry.  The counter
+// holds exactly n once its GEMM is complete (its slot is not reused in the same
+// launch), so a value past n means a miscount: it would have released this wait
+// early, and it is recorded in *status.
+__device__ __forceinline__ bool counter_wait(const unsigned int *c, unsigned int n, int *status) {
   const unsigned long long t0 = gtime();
   for (int i = 0;; ++i) {
-    if (counter_reached(c, n)) return true;
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(c) : "memory");
+    if ((int)(v - n) >= 0) {
+      if (v != n) set_status(status, DFLOW_ERR_BAD_STATE);
+      return true;
+    }
     if ((i & 15) == 15 && gtime() - t0 > WAIT_NS) return false;
   }
 }
@@ -1010,7 +1013,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
             // the launch's inputs: once, before this producer's first copy
             if (!dep_done) dep_wait(p.dep, p.status);
             dep_done = true;
-          } else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n)) {
+          } else if (!counter_wait(p.g[j - 1].done, p.g[j - 1].done_n, p.status)) {
             ok = false;
             break;
           }
@@ -1111,7 +1114,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       if (leader) {
         if (j == 0)
           dep_wait(p.dep, p.status);
-        else if (!p.independent && !counter_wait(p.g[j - 1].done, p.g[j - 1].done_n))
+        else if (!p.independent && !counter_wait(p.g[j - 1].done, p.g[j - 1].done_n, p.status))
           set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
       }
       epi_bar();
@@ -1149,12 +1152,8 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         // a leftover part counts for the owner that completed its columns
         if (leader) finished += ti >= 0 || sm.left_last ? 1u : 0u;
       }
-      // this CTA's share of GEMM j is written (a barrier over the epilogue threads above);
-      // a count past the GEMM's target would release a later wait on this counter early
-      if (ok && leader && finished > 0) {
-        const unsigned int old = atom_add_acq_rel(g.done, finished);
-        if ((int)(old + finished - g.done_n) > 0) set_status(p.status, DFLOW_ERR_BAD_STATE);
-      }
+      // this CTA's share of GEMM j is written (a barrier over the epilogue threads above)
+      if (ok && leader && finished > 0) counter_add(g.done, finished);
     }
     if (!ok && leader) {
       set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);

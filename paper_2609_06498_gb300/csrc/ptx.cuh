@@ -183,7 +183,12 @@ __device__ __forceinline__ void dep_wait(const Dep &d, int *status) {
   for (int i = 0;; ++i) {
     unsigned int v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(d.wait) : "memory");
-    if ((int)(v - d.wait_n) >= 0) return;
+    if ((int)(v - d.wait_n) >= 0) {
+      // the previous launch's counter holds exactly its target once it is done:
+      // more is a miscount that would have released this wait early
+      if (v != d.wait_n) atomicCAS(status, 0, (int)DFLOW_ERR_BAD_STATE);
+      return;
+    }
     if ((i & 15) == 15 && gtime() - t0 > WAIT_NS) {
       atomicCAS(status, 0, (int)DFLOW_ERR_DEVICE_TIMEOUT);
       return;
