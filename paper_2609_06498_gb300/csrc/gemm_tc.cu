@@ -46,6 +46,7 @@ constexpr int BK = 64;            // k elements per k-block (128 bytes of bf16: 
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int MAX_NPAD = 256;
 constexpr int MAX_SPLIT_NPAD = 64;  // split-K (P > 1) only for up to 64 token columns
+constexpr int SEQ_MAX_NPAD = 128;   // token columns of the persistent layer-segment kernel
 constexpr int THREADS = 192;
 constexpr int SMEM_BUDGET = 224 * 1024;
 
@@ -421,7 +422,7 @@ __device__ __forceinline__ unsigned int atom_add_acq_rel(unsigned int *a, unsign
 // CW4 > 0: the split is 4-way over npad = 4 CW4 columns (each owner finishes
 // CW4 of them), known at compile time: every loop has a fixed trip count, the
 // owner of a column group is a constant, and the epilogue covers CW4 columns.
-// lp.acc set (CW4 > 0 only): the cluster holds one part of the tile; each owner
+// lp.acc set (0 < CW4 <= 16 only): the cluster holds one part of the tile; each owner
 // stores its columns' sum in its part's slot, and only the one completing the
 // count adds the parts (in part order, so the result does not depend on the
 // arrival order) and runs their epilogue (sm.left_last = 1 in that CTA).
@@ -430,8 +431,8 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
                                             uint32_t lane_addr, int i, int t, int r, int sub, int lane, int rr,
                                             int rbase, bool leader, uint32_t next_bytes, uint32_t rfree_n,
                                             const LeftPart lp = LeftPart{}) {
-  static_assert(CW4 % 4 == 0 && CW4 <= 16, "owner width");
-  constexpr int NC = CW4 ? CW4 : 16;  // epilogue columns per chunk
+  static_assert(CW4 % 4 == 0 && CW4 <= 32, "owner width");
+  constexpr int NC = CW4 > 0 && CW4 < 16 ? CW4 : 16;  // epilogue columns per chunk
   const int P = CW4 ? 4 : P_, npad = CW4 ? 4 * CW4 : npad_;
   const int w4 = CW4 ? CW4 : splitk_w4(M, P);
   const int s0 = min(rr * w4, M), s1 = min((rr + 1) * w4, M);
@@ -523,7 +524,7 @@ __device__ __forceinline__ bool splitk_tile(const PT &g, Smem &sm, float *rx, in
         released = true;
       }
       if (c0 > s0) epilogue_prefetch<EP, PT, NC>(g, sm, t, r, c0, min(NC, s1 - c0), pre);
-      if constexpr (CW4 > 0) {
+      if constexpr (CW4 > 0 && CW4 <= 16) {
         if (lp.acc != nullptr) {
           // one chunk (CW4 <= 16): this cluster's part of the columns into its slot
           const size_t slot = (size_t)BM * npad;
@@ -896,8 +897,8 @@ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
   return t;
 }
 // bytes this CTA receives in a split-K tile of GEMM j
-__device__ __forceinline__ uint32_t seq_recv_bytes(int M, int rank) {
-  const int w4 = splitk_w4(M, SEQ_P);
+__device__ __forceinline__ uint32_t seq_recv_bytes(int M, int npad, int rank) {
+  const int w4 = npad / SEQ_P;
   return splitk_recv_bytes(SEQ_P, min(rank * w4, M), min((rank + 1) * w4, M));
 }
 // true when this CTA has another tile after tile ti of GEMM j (ti = -1: its leftover part)
@@ -911,7 +912,9 @@ __device__ __forceinline__ bool seq_more(const SeqTab &tb, int j, int ti) {
 // one tile of GEMM g (split-K over the SEQ_P CTAs of the cluster, NPAD token
 // columns); false when a bounded wait expired.  rfree counts SEQ_P - 1
 // arrivals per tile, one from each other owner.
-// lt >= 0: t is leftover tile lt, the cluster holds one part of it.
+// lt >= 0: t is leftover tile lt, the cluster holds one part of it (the host
+// splits tiles over clusters only for NPAD <= MAX_SPLIT_NPAD: one epilogue chunk
+// per owner).
 template <int EP, int NPAD>
 __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, uint32_t lane_addr, int i, int t, int lt,
                                          int part, int r, int sub, int lane, int rank, bool leader,
@@ -936,7 +939,7 @@ constexpr int SEQ_THREADS = THREADS + 32;  // warp 6: the activation producer
 // the CTA's schedule in shared memory, after the Smem block
 constexpr size_t SEQ_SMEM_TAB_OFF = (sizeof(Smem) + 15) & ~(size_t)15;
 
-// NPAD: the token columns padded to 16 (p.npad), a compile-time constant so that
+// NPAD: the token columns (p.npad, seq_npad), a compile-time constant so that
 // the split-K epilogue has fixed trip counts
 template <int NPAD>
 __global__ void __launch_bounds__(SEQ_THREADS, 1)
@@ -974,7 +977,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
     const SeqTab tb = *stab;
     bool any = false;
     for (int j = 0; j < tb.n; ++j) any = any || sel4(tb.nt, j) > 0 || sel4(tb.lt, j) >= 0;
-    mbar_expect_tx(&sm.recv, any ? seq_recv_bytes(p.M, rank) : 0u);
+    mbar_expect_tx(&sm.recv, any ? seq_recv_bytes(p.M, NPAD, rank) : 0u);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
@@ -1131,7 +1134,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         const int t = ti < 0 ? g.Tf + lt : sel4(tb.t0, j) + ti * sel4(tb.dt, j);
         const int tl = ti < 0 ? lt : -1;
         const int fp = ti < 0 ? sel4(tb.lpart, j) : 0;  // the cluster's part of its leftover tile
-        const uint32_t nb = seq_more(tb, j, ti) ? seq_recv_bytes(p.M, rank) : 0u;
+        const uint32_t nb = seq_more(tb, j, ti) ? seq_recv_bytes(p.M, NPAD, rank) : 0u;
         switch (g.mode) {
           case EP_RESID:
             ok = seq_tile<EP_RESID, NPAD>(g, sm, rx, lane_addr, i, t, tl, fp, r, sub, lane, rank, leader, nb);
@@ -1313,13 +1316,16 @@ size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
 
 // clusters of SEQ_P persistent CTAs that are resident at once
 using SeqKernel = void (*)(SeqMaps, SeqParams);
-// the instantiation for npad token columns (16, 32, 48 or 64), or null
+// the instantiation for npad token columns (seq_npad), or null
 SeqKernel seq_kernel(int npad) {
   switch (npad) {
     case 16: return k_gemm_seq<16>;
     case 32: return k_gemm_seq<32>;
     case 48: return k_gemm_seq<48>;
     case 64: return k_gemm_seq<64>;
+    case 80: return k_gemm_seq<80>;
+    case 96: return k_gemm_seq<96>;
+    case 128: return k_gemm_seq<128>;
     default: return nullptr;
   }
 }
@@ -1506,8 +1512,15 @@ static bool seq_left_enabled() {
   return on;
 }
 
+// token columns of the persistent kernel for M rows: M rounded up to 16, and
+// 112 up to 128 (one instantiation fewer; the extra columns are zero rows of X)
+static int seq_npad(int M) {
+  const int n = (M + 15) / 16 * 16;
+  return n == 112 ? 128 : n;
+}
+
 bool seq_supported(int M) {
-  return M >= 1 && (M + 15) / 16 * 16 <= MAX_SPLIT_NPAD && encode_fn() != nullptr;
+  return M >= 1 && seq_npad(M) <= SEQ_MAX_NPAD && encode_fn() != nullptr;
 }
 
 // two Q/K/V epilogues build the same column table (positions and pool slots)
@@ -1525,7 +1538,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   p.n = n;
   p.independent = independent ? 1 : 0;
   p.M = M;
-  p.npad = (M + 15) / 16 * 16;
+  p.npad = seq_npad(M);
   p.status = status;
   int cols = 32;
   while (cols < 2 * p.npad) cols <<= 1;
@@ -1550,12 +1563,13 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
     g.T = (q.N + BM - 1) / BM;
     g.kb = q.K / BK;
     g.mode = mode;
-    // leftover tiles when they divide the clusters evenly and every part keeps a k-block
+    // leftover tiles when they divide the clusters evenly and every part keeps a
+    // k-block (up to 64 columns: one epilogue chunk per owner)
     const int lo = g.T % p.Q;
     g.Tf = g.T;
     g.Tl = 0;
     g.ls = 1;
-    if (lo > 0 && p.Q <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
+    if (lo > 0 && p.npad <= MAX_SPLIT_NPAD && p.Q <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
         seq_left_enabled()) {
       g.Tf = g.T - lo;
       g.Tl = lo;

@@ -13,6 +13,8 @@ pytestmark = pytest.mark.gpu
 SHAPES = [  # (N, K, M)
     (256, 64, 1), (1000, 512, 17), (6144, 4096, 17), (4096, 4096, 32), (24576, 4096, 17), (4096, 12288, 17),
     (151936, 4096, 17), (2048, 4096, 272), (512, 1472, 48), (384, 3072, 300), (2944, 512, 5),
+    # persistent kernel above 64 columns: two epilogue chunks per owner (68 -> 80, 100 -> 128 columns)
+    (6144, 2560, 68), (2560, 9728, 100), (4096, 4096, 128),
 ]
 
 
@@ -39,6 +41,12 @@ def _rel(a, b):
     return float((a - b).abs().max() / b.abs().max())
 
 
+def _tol(K):
+    # both sides accumulate K products in fp32: rounding walks like sqrt(K) u
+    # (u = 2^-24) of the largest output on each side; 4 sqrt(K) u, 1e-5 at least
+    return max(1e-5, 4 * K ** 0.5 * 2.0 ** -24)
+
+
 @pytest.mark.parametrize("path", [1, 0], ids=["tcgen05", "simt"])
 @pytest.mark.parametrize("N,K,M", SHAPES)
 def test_store_and_resid(eng, path, N, K, M):
@@ -50,7 +58,7 @@ def test_store_and_resid(eng, path, N, K, M):
     eng.debug_gemm(path, W, X, 0, out, st)
     torch.cuda.synchronize()
     assert int(st) == 0
-    assert _rel(out, ref) < 1e-5
+    assert _rel(out, ref) < _tol(K)
     base = torch.randn(M, N, device="cuda")
     acc = base.clone()
     eng.debug_gemm(path, W, X, 1, acc, st)
@@ -63,7 +71,7 @@ def test_store_and_resid(eng, path, N, K, M):
 
 
 @pytest.mark.parametrize("path", [1, 0], ids=["tcgen05", "simt"])
-@pytest.mark.parametrize("N,K,M", [(2944, 512, 17), (24576, 4096, 17), (3072, 1024, 300)])
+@pytest.mark.parametrize("N,K,M", [(2944, 512, 17), (24576, 4096, 17), (19456, 2560, 68), (3072, 1024, 300)])
 def test_swiglu_and_silu(eng, path, N, K, M):
     W, X, ref = _inputs(N, K, M, 7 * N + M)
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
