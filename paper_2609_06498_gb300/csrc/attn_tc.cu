@@ -443,7 +443,8 @@ cudaError_t launch(const CUtensorMap &tm, const Dims &D, int batch, const AttnAr
 // ===========================================================================
 constexpr int T5_ROWS = 128;     // query rows per CTA (MMA M)
 constexpr int T5_STAGES = 4;     // K/V pages in flight
-constexpr int T5_SPLITS = 8;     // key splits = cluster size; split s takes pages s, s + 8, ...
+// key splits = cluster size S (8, or 4 when 8 would not fit in one wave); split s
+// takes pages s, s + S, ...
 constexpr float T5_TAU = 8.0f;   // rescale threshold, log2 units
 constexpr int T5_TMEM_COLS = 256;  // O: 128 columns, S: two buffers of 64
 
@@ -505,14 +506,15 @@ __device__ __forceinline__ uint64_t smem_desc_mn(uint32_t saddr, uint32_t lbo) {
   d |= (uint64_t)2 << 61;
   return d;
 }
-// pages of split s: s, s + T5_SPLITS, ...; the ones below n_tiles hold keys
+// pages of split s: s, s + S, ...; the ones below n_tiles hold keys
+template <int S>
 __device__ __forceinline__ int t5_pool_tiles(int n_tiles, int split) {
-  return n_tiles > split ? (n_tiles - 1 - split) / T5_SPLITS + 1 : 0;
+  return n_tiles > split ? (n_tiles - 1 - split) / S + 1 : 0;
 }
 
 // q_tma: the CTA's query rows arrive as two boxes of the 3D map tq over
 // [rows][hq][128] (64 dims x G heads x R rows); else each softmax thread loads its row
-template <bool BLOCK>
+template <bool BLOCK, int S>
 __global__ void __launch_bounds__(THREADS, 1)
 k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tq, Dims D, AttnArgs a,
           int q_tma, int *status) {
@@ -530,7 +532,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   float *o_sm = reinterpret_cast<float *>(ring);  // [128][128] fp32 after the key loop
 
   const int kvh = blockIdx.x, b = blockIdx.y;
-  const int split = blockIdx.z % T5_SPLITS, qg = blockIdx.z / T5_SPLITS;
+  const int split = blockIdx.z % S, qg = blockIdx.z / S;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int G = D.hq / D.hkv, R = D.R, QR = R * G, row0 = qg * T5_ROWS;
   const int *pt = a.page_table + (size_t)b * D.pages_per_seq;
@@ -557,11 +559,11 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   };
   if (warp == 0) {
     // page ids of this split's first 32 pages
-    const int t = split + T5_SPLITS * lane;
+    const int t = split + S * lane;
     pg = t < D.pages_per_seq ? __ldg(pt + t) : 0;
     const int n_old = a.causal ? nk - R : nk;  // pool keys older than this round's block
-    n_pre = min(t5_pool_tiles((nk + 63) / 64, split), T5_STAGES);
-    while (n_early < n_pre && (split + T5_SPLITS * n_early + 1) * 64 <= n_old) ++n_early;
+    n_pre = min(t5_pool_tiles<S>((nk + 63) / 64, split), T5_STAGES);
+    while (n_early < n_pre && (split + S * n_early + 1) * 64 <= n_old) ++n_early;
     if (lane == 0) {
       prefetch_tensormap(&tm);
       if (q_tma) prefetch_tensormap(&tq);
@@ -600,8 +602,8 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   const uint32_t t_o = tmem, t_s = tmem + 128;
   const int n_keys = sm.n_keys;
   const int n_tiles = (n_keys + 63) / 64;
-  const int Tp = t5_pool_tiles(n_tiles, split);
-  const int T = Tp + ((BLOCK && split == T5_SPLITS - 1) ? 1 : 0);
+  const int Tp = t5_pool_tiles<S>(n_tiles, split);
+  const int T = Tp + ((BLOCK && split == S - 1) ? 1 : 0);
 
   if (warp == 0) {
     // the projection's outputs: Q, then the first pages that hold block rows
@@ -629,7 +631,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
       const int stage = it % T5_STAGES;
       const uint32_t ph = (it / T5_STAGES) & 1;
       if ((it & 31) == 0) {
-        const int t = split + T5_SPLITS * (it + lane);
+        const int t = split + S * (it + lane);
         pg = (it + lane < Tp) ? pt[t] : 0;
       }
       const int page = __shfl_sync(0xffffffffu, pg, it & 31);
@@ -765,7 +767,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
     for (int i = 0; i < T; ++i) {
       const int buf = i & 1, stage = i % T5_STAGES;
       const bool blk = i >= Tp;
-      const int tile = split + T5_SPLITS * i;
+      const int tile = split + S * i;
       if (!wait_all(&sm.s_full[buf], (uint32_t)((i >> 1) & 1))) { ok = false; break; }
       tc_fence_after();
       float s[64];
@@ -885,19 +887,19 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   __syncthreads();
   cluster_sync();
   const int n_valid = min(QR - row0, T5_ROWS);
-  const int rpc = (n_valid + T5_SPLITS - 1) / T5_SPLITS;
+  const int rpc = (n_valid + S - 1) / S;
   const int r_lo = split * rpc, nr = max(min(r_lo + rpc, n_valid) - r_lo, 0);
   const int units = nr * (HD / 4);
-  // one round trip of remote loads: thread t < 8 nr takes (row t / 8, split t % 8)'s
-  // max and sum; every thread takes the 8 split partials of up to two
+  // one round trip of remote loads: thread t < S nr takes (row t / S, split t % S)'s
+  // max and sum; every thread takes the S split partials of up to two
   // (row, 4-dim chunk) units
   float mv = -INFINITY, lv = 0.f;
-  if (threadIdx.x < nr * T5_SPLITS) {
-    const int rr = r_lo + threadIdx.x / T5_SPLITS, sp = threadIdx.x % T5_SPLITS;
+  if (threadIdx.x < nr * S) {
+    const int rr = r_lo + threadIdx.x / S, sp = threadIdx.x % S;
     mv = ld_dsmem_f32(mapa(smem_u32(sm.m + rr), (uint32_t)sp));
     lv = ld_dsmem_f32(mapa(smem_u32(sm.l + rr), (uint32_t)sp));
   }
-  float4 x[2][T5_SPLITS];
+  float4 x[2][S];
   auto load_units = [&](int u0) {
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -906,23 +908,23 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
         const int rr = r_lo + u / (HD / 4), c4 = u % (HD / 4);
         const int off = rr * HD + ((c4 ^ (rr & 7)) << 2);
 #pragma unroll
-        for (int sp = 0; sp < T5_SPLITS; ++sp) x[h][sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + off), (uint32_t)sp));
+        for (int sp = 0; sp < S; ++sp) x[h][sp] = ld_dsmem_f4(mapa(smem_u32(o_sm + off), (uint32_t)sp));
       }
     }
   };
   load_units(threadIdx.x);
-  // merge weight of (row, split): 2^(m - M) / sum_s 2^(m_s - M) l_s over the 8
+  // merge weight of (row, split): 2^(m - M) / sum_s 2^(m_s - M) l_s over the S
   // lanes of the row (the Q tile is free now and holds them)
-  float *wsm = reinterpret_cast<float *>(qs);  // [rpc][T5_SPLITS]
+  float *wsm = reinterpret_cast<float *>(qs);  // [rpc][S]
   {
     float M = mv;
 #pragma unroll
-    for (int o = 1; o < T5_SPLITS; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    for (int o = 1; o < S; o <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
     const float c = mv == -INFINITY ? 0.f : exp2f(mv - M);
     float L = c * lv;
 #pragma unroll
-    for (int o = 1; o < T5_SPLITS; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    if (threadIdx.x < nr * T5_SPLITS) wsm[threadIdx.x] = L > 0.f ? c / L : 0.f;
+    for (int o = 1; o < S; o <<= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (threadIdx.x < nr * S) wsm[threadIdx.x] = L > 0.f ? c / L : 0.f;
   }
   __syncthreads();
   bf16 *out = static_cast<bf16 *>(a.out);
@@ -935,8 +937,8 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
       const int rl = u / (HD / 4), d4 = (u % (HD / 4)) * 4, q_r = row0 + r_lo + rl;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int sp = 0; sp < T5_SPLITS; ++sp) {
-        const float c = wsm[rl * T5_SPLITS + sp];
+      for (int sp = 0; sp < S; ++sp) {
+        const float c = wsm[rl * S + sp];
         acc.x += c * x[h][sp].x;
         acc.y += c * x[h][sp].y;
         acc.z += c * x[h][sp].z;
@@ -956,24 +958,42 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   }
 }
 
-template <bool BLOCK>
-cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs a, int *status, cudaStream_t s,
-                      DepChain *chain) {
-  const size_t smem = 1024 + 2 * T5_ROWS * 128 + T5_STAGES * 2 * (64 * 128 * 2) + 2 * T5_ROWS * 128 + sizeof(T5Smem);
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_attn_t5<BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    attr = true;
+// resident clusters of S CTAs of k_attn_t5<BLOCK, S> (0 when the query fails)
+template <bool BLOCK, int S>
+int t5_resident_clusters(size_t smem) {
+  static int n = -1;
+  if (n >= 0) return n;
+  n = 0;
+  if (cudaFuncSetAttribute(k_attn_t5<BLOCK, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) ==
+      cudaSuccess) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(S);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = S;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, k_attn_t5<BLOCK, S>, &cfg) != cudaSuccess) n = 0;
   }
+  cudaGetLastError();
+  return n;
+}
+
+template <bool BLOCK, int S>
+cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs a, int *status, cudaStream_t s,
+                      DepChain *chain, size_t smem) {
   const int G = D.hq / D.hkv;
   const int qgroups = (D.R * G + T5_ROWS - 1) / T5_ROWS;
   // one group of query rows: they arrive as two 3D boxes (64 dims x G heads x R rows)
   CUtensorMap tq{};
   const int q_tma = (qgroups == 1 && tensor_map_3d(&tq, a.q, D.hd, D.hq, batch * D.R, G, D.R)) ? 1 : 0;
-  a.dep = chain ? chain->take((unsigned)(D.hkv * batch * T5_SPLITS * qgroups)) : Dep{};
+  a.dep = chain ? chain->take((unsigned)(D.hkv * batch * S * qgroups)) : Dep{};
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(D.hkv, batch, T5_SPLITS * qgroups);
+  cfg.gridDim = dim3(D.hkv, batch, S * qgroups);
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
@@ -983,10 +1003,25 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs 
   at[1].id = cudaLaunchAttributeClusterDimension;
   at[1].val.clusterDim.x = 1;
   at[1].val.clusterDim.y = 1;
-  at[1].val.clusterDim.z = T5_SPLITS;
+  at[1].val.clusterDim.z = S;
   cfg.attrs = at;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK>, tm, tq, D, a, q_tma, status);
+  return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK, S>, tm, tq, D, a, q_tma, status);
+}
+
+// eight key splits per (kv head, sequence, query group), or four when the
+// eight-CTA clusters would need a second wave and the four-CTA ones fit in one
+// (the per-CTA key loop is latency bound: one wave of twice the pages is shorter)
+template <bool BLOCK>
+cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
+                          cudaStream_t s, DepChain *chain) {
+  const size_t smem = 1024 + 2 * T5_ROWS * 128 + T5_STAGES * 2 * (64 * 128 * 2) + 2 * T5_ROWS * 128 + sizeof(T5Smem);
+  const int G = D.hq / D.hkv;
+  const long long units = (long long)D.hkv * batch * ((D.R * G + T5_ROWS - 1) / T5_ROWS);
+  const int r8 = t5_resident_clusters<BLOCK, 8>(smem), r4 = t5_resident_clusters<BLOCK, 4>(smem);
+  if (r8 < 1) return cudaErrorInvalidValue;
+  if (units > r8 && units <= r4) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
+  return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
 }
 
 }  // namespace
@@ -1004,8 +1039,8 @@ cudaError_t attention_tc(const Dims &D, int batch, const AttnArgs &a_in, int *st
   if (!tensor_map(&tm, a.pool, rows, D.hd, D.hd, 64)) return cudaErrorInvalidValue;
   const bool block = !a.causal;
   if (D.hd == 128 && getenv("DFLOW_MMA_SYNC_ATTENTION") == nullptr)
-    return block ? launch_t5<true>(tm, D, batch, a, status, s, chain)
-                 : launch_t5<false>(tm, D, batch, a, status, s, chain);
+    return block ? launch_t5_any<true>(tm, D, batch, a, status, s, chain)
+                 : launch_t5_any<false>(tm, D, batch, a, status, s, chain);
   if (chain) chain->brk();
   if (D.hd == 128) return block ? launch<128, true>(tm, D, batch, a, status, s) : launch<128, false>(tm, D, batch, a, status, s);
   return block ? launch<64, true>(tm, D, batch, a, status, s) : launch<64, false>(tm, D, batch, a, status, s);
