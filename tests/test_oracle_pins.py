@@ -4,6 +4,7 @@ No test here retypes an oracle formula: each one checks a closed form worked by
 hand, a library routine, an invariant, or a brute-force recomputation.
 """
 import math
+from pathlib import Path
 
 import numpy as np
 import pytest
@@ -188,16 +189,22 @@ def test_feature_projection_selects_layer_outputs(tiny_w):
 # ---------------------------------------------------------------------------
 
 
-@pytest.mark.parametrize("block,g,a,committed", [
-    # no proposal matches: a = 0, bonus = g[0]
-    ([7, 1, 2, 3], [9, 8, 8, 8], 0, [9, -1, -1, -1]),
-    # first two match (y1 == g0, y2 == g1), third does not
-    ([7, 1, 2, 3], [1, 2, 5, 6], 2, [1, 2, 5, -1]),
-    # all match: bonus is the prediction after the last draft
-    ([7, 1, 2, 3], [1, 2, 3, 4], 3, [1, 2, 3, 4]),
-    # a later match after a mismatch does not count
-    ([7, 1, 2, 3], [0, 2, 3, 4], 0, [0, -1, -1, -1]),
-])
+GOLDEN = Path(__file__).parent / "golden"
+
+
+def _golden_lines(name):
+    return [ln for ln in (GOLDEN / name).read_text().splitlines() if ln.strip() and not ln.startswith("#")]
+
+
+def _accept_cases():
+    cases = []
+    for ln in _golden_lines("accept_eq3_hand_cases.txt"):
+        block, g, a, committed = (f.split() for f in ln.split("|"))
+        cases.append(([int(x) for x in block], [int(x) for x in g], int(a[0]), [int(x) for x in committed]))
+    return cases
+
+
+@pytest.mark.parametrize("block,g,a,committed", _accept_cases())
 def test_accept_partition_hand_cases(block, g, a, committed):
     cfg, o = _micro_oracle()
     cfg = cfg.replace(block=3)
@@ -411,8 +418,11 @@ def test_draft_reads_context_features_up_to_n_minus_2(tiny_oracle):
 
 
 def test_splitmix64_published_vector():
-    # first output of SplitMix64 seeded with 0 (Steele et al. reference implementation)
-    assert synth.splitmix64(0) == 0xE220A8397B1DCDAF
+    # the generator's i-th output is the finaliser applied to state i * gamma
+    gamma = 0x9E3779B97F4A7C15
+    want = [int(h, 16) for h in _golden_lines("splitmix64_seed0.txt")]
+    assert len(want) == 4
+    assert [synth.splitmix64((i * gamma) % 2 ** 64) for i in range(4)] == want
 
 
 def test_schedules():
