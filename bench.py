@@ -306,6 +306,7 @@ def main():
         cfg = cfg.replace(n_layers=args.depth, draft_layers=min(cfg.draft_layers, args.depth),
                           feat_layers=tuple(sorted({1, args.depth})))
     K, Wm = args.steps, args.warmup
+    relay = bool(args.relay)  # 0: the DFlash baseline (mask embeddings only, nothing carried)
     n_rounds = Wm + K
     lens = synth.prompt_lengths(cfg)
     max_ctx = cfg.replace(new_tokens=n_rounds * cfg.rows).max_ctx()
@@ -322,7 +323,7 @@ def main():
     comm = torch.empty(cfg.batch, cfg.rows, dtype=torch.int32, device="cuda")
 
     for w in range(Wm):
-        eng.round(st, forced_dev[w], out=(acc, comm))
+        eng.round(st, forced_dev[w], relay=relay, out=(acc, comm))
     torch.cuda.synchronize()
     # snapshot of the per-sequence state after warmup: every leg starts from it
     snap = {k: getattr(st, k).clone() for k in ("tokens", "seq_len", "carry", "n_carry", "boundary")}
@@ -341,7 +342,7 @@ def main():
         # rounds inside a profiler range, for `ncu --profile-from-start off`
         torch.cuda.cudart().cudaProfilerStart()
         for k in range(min(K, 2)):
-            eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+            eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
         torch.cuda.synchronize()
         torch.cuda.cudart().cudaProfilerStop()
         print(json.dumps({"profile_only": True, "launches": eng.launch_count()}))
@@ -360,7 +361,7 @@ def main():
         barrier()
         ev[0].record(stream)
         for k in range(K):
-            eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+            eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
             ev[k + 1].record(stream)
         torch.cuda.synchronize()
     launches = eng.launch_count() - n0
@@ -382,7 +383,7 @@ def main():
         e0.record(stream)
         for k in range(K):
             d_forced.copy_(h_forced[Wm + k], non_blocking=True)
-            eng.round(st, d_forced, out=(acc, comm))
+            eng.round(st, d_forced, relay=relay, out=(acc, comm))
             h_acc[k].copy_(acc, non_blocking=True)
             h_comm[k].copy_(comm, non_blocking=True)
         e1.record(stream)
@@ -393,6 +394,7 @@ def main():
                "h2d_bytes_per_step": 4 * cfg.batch, "d2h_bytes_per_step": 4 * cfg.batch * (1 + cfg.rows)}
 
     # ---- per-step split: the round's four calls one at a time, events between them
+    # (the per-call entry points draft and carry with the relay on)
     restore()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
     for k in range(K):
@@ -416,7 +418,7 @@ def main():
     restore()
     eng.profile(True)
     for k in range(K):
-        eng.round(st, forced_dev[Wm + k], out=(acc, comm))
+        eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
     torch.cuda.synchronize()
     prof = eng.profile_read()
     eng.profile(False)
