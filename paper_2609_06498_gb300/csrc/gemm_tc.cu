@@ -1545,6 +1545,12 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   p.tmem_cols = cols;
   const size_t smem = seq_smem(p.npad, &p.stages, &p.rx_bytes);
   p.Q = seq_clusters(p.npad, smem);
+  // DFLOW_SEQ_CLUSTERS=n caps the grid at n clusters (all still resident at once)
+  static const int q_cap = [] {
+    const char *e = getenv("DFLOW_SEQ_CLUSTERS");
+    return e ? atoi(e) : 0;
+  }();
+  if (q_cap > 0 && q_cap < p.Q) p.Q = q_cap;
   if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
   const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   for (int j = 0; j < n; ++j) {
