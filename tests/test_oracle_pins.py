@@ -130,6 +130,126 @@ def test_zero_blocks_leave_embedding_in_residual():
 
 
 # ---------------------------------------------------------------------------
+# Qwen3 attention inputs: per-head q/k RMSNorm (with its gains) comes first,
+# the rotary embedding last; the drafter's context keys/values (Sec. 3: target
+# features injected into the K and V projections) follow the same order with no
+# input norm.  Hand values use head_dim 2, where the rotary embedding at
+# position p is multiplication of (x0 + i x1) by e^{ip} (theta^0 = 1).
+# ---------------------------------------------------------------------------
+
+
+def _rot(x0, x1, p):
+    z = complex(x0, x1) * complex(math.cos(p), math.sin(p))
+    return [z.real, z.imag]
+
+
+def _attn_micro(**over):
+    f32 = lambda rows: np.array(rows, np.float32)  # noqa: E731
+    w = {
+        "t0.wq": f32([[3, 0, 0, 0], [0, 4, 0, 0], [0, 0, 1, 0], [0, 0, 0, -2]]),
+        "t0.wk": f32([[0, 0, 2, 0], [0, 0, 0, 1]]),
+        "t0.wv": f32([[1, 1, 0, 0], [0, 0, 1, 1]]),
+        "t0.q_norm": f32([1, 2]),
+        "t0.k_norm": f32([0.5, 3]),
+        "embed": f32([[0, 0, 0, 0], [10, 10, 10, 10], [-5, -5, -5, -5], [0, 0, 0, 0], [0, 0, 0, 0]]),
+    }
+    w.update(over)
+    return _micro_oracle(**w)
+
+
+def test_qk_rmsnorm_with_gains_then_rotary_hand_values():
+    cfg, o = _attn_micro()
+    # h = RMSNorm(10, 10, 10, 10) = (1, 1, 1, 1): q head 0 = (3, 4), head 1 = (1, -2), k = (2, 1)
+    q, k, v = o._qkv("t0.", np.full((1, 4), 10.0), np.array([5]))
+    r0, r1, rk = math.sqrt(12.5), math.sqrt(2.5), math.sqrt(2.5)
+    want_q0 = _rot(3 / r0 * 1, 4 / r0 * 2, 5)  # normalised, gains (1, 2), then rotated by 5 rad
+    want_q1 = _rot(1 / r1 * 1, -2 / r1 * 2, 5)
+    want_k = _rot(2 / rk * 0.5, 1 / rk * 3, 5)  # gains (0.5, 3)
+    assert np.allclose(q[0, 0], want_q0, atol=1e-6)
+    assert np.allclose(q[0, 1], want_q1, atol=1e-6)
+    assert np.allclose(k[0, 0], want_k, atol=1e-6)
+    assert np.allclose(v[0, 0], [2, 2], atol=1e-6)  # values: no norm, no rotation
+
+
+def test_target_cache_keys_hand_values_at_their_positions():
+    # W_o = W_d = 0 keep the residual at the embedding; tokens 1 and 2 have
+    # RMSNorm(E) = (1, 1, 1, 1) and (-1, -1, -1, -1); written at positions 3 and 4
+    cfg, o = _attn_micro()
+    st = o.new_state(cap=16)
+    o.target_forward(st, 0, [1, 2], 3)
+    rk = math.sqrt(2.5)
+    assert np.allclose(st.k[0, 0, 3, 0], _rot(1 / rk, 3 / rk, 3), atol=1e-6)
+    assert np.allclose(st.k[0, 0, 4, 0], _rot(-1 / rk, -3 / rk, 4), atol=1e-6)
+    assert np.allclose(st.v[0, 0, 3, 0], [2, 2], atol=1e-6)
+    assert np.allclose(st.v[0, 0, 4, 0], [-2, -2], atol=1e-6)
+    assert not st.k[0, 0, :3].any() and not st.k[0, 0, 5:].any()
+
+
+def test_qk_scores_depend_only_on_relative_offset(tiny_oracle):
+    """RoPE's defining property holds for the projected q/k only if the rotation
+    is applied after the per-head norm (the gains are not rotation invariant)."""
+    o = tiny_oracle
+    assert np.ptp(o.W["t0.q_norm"]) > 0.1 and np.ptp(o.W["t0.k_norm"]) > 0.1
+    x = np.random.default_rng(11).normal(size=(2, TINY.d))
+    qa, _, _ = o._qkv("t0.", x[:1], np.array([37]))
+    _, ka, _ = o._qkv("t0.", x[1:], np.array([30]))
+    qb, _, _ = o._qkv("t0.", x[:1], np.array([1037]))
+    _, kb, _ = o._qkv("t0.", x[1:], np.array([1030]))
+    sa = np.einsum("hd,kd->hk", qa[0], ka[0])
+    sb = np.einsum("hd,kd->hk", qb[0], kb[0])
+    assert np.allclose(sa, sb, atol=1e-9)
+
+
+def test_target_keys_and_logits_invariant_to_qk_projection_scale(tiny_w):
+    """Per-head RMSNorm on q and k removes the scale of W_q and W_k (up to eps)."""
+    prompt = synth.prompts(TINY)[0][:12]
+    o = Oracle(TINY, tiny_w)
+    st = o.new_state()
+    lg, _ = o.target_forward(st, 0, prompt, 0)
+    W = dict(tiny_w)
+    for l in range(TINY.n_layers):
+        W[f"t{l}.wq"] = W[f"t{l}.wq"] * 4.0
+        W[f"t{l}.wk"] = W[f"t{l}.wk"] * 4.0
+    o2 = Oracle(TINY, W)
+    st2 = o2.new_state()
+    lg2, _ = o2.target_forward(st2, 0, prompt, 0)
+    # eps 1e-6 against mean squares near 0.1 leaves about 1e-5 of the scale
+    k1, k2 = st.k[:, 0, :12], st2.k[:, 0, :12]
+    assert np.abs(k1 - k2).max() < 1e-4 * np.abs(k1).max()
+    assert np.abs(lg - lg2).max() < 1e-4 * np.abs(lg).max()
+
+
+def test_context_kv_injection_hand_values():
+    """Sec. 3: feature f at position p enters draft layer l as
+    k = RoPE(k_norm(W_k f), p), v = W_v f (f is RMSNormed by Eq. 1 already)."""
+    f32 = lambda rows: np.array(rows, np.float32)  # noqa: E731
+    cfg, o = _micro_oracle(**{"d0.wk": f32([[1, 0, 0, 0], [0, 1, 0, 0]]), "d0.wv": f32([[0, 0, 0, 1], [1, 1, 0, 0]]),
+                              "d0.k_norm": f32([2, 0.5])})
+    st = o.new_state(cap=16)
+    feats = np.array([[1.0, 2.0, 0.0, -1.0], [-3.0, 1.0, 5.0, 2.0]])
+    o.ctx_append(st, 0, feats, 7)
+    r1, r2 = math.sqrt(2.5), math.sqrt(5.0)  # RMS of (1, 2) and of (-3, 1)
+    assert np.allclose(st.dk[0, 0, 7, 0], _rot(1 / r1 * 2, 2 / r1 * 0.5, 7), atol=1e-6)
+    assert np.allclose(st.dk[0, 0, 8, 0], _rot(-3 / r2 * 2, 1 / r2 * 0.5, 8), atol=1e-6)
+    assert np.allclose(st.dv[0, 0, 7, 0], [-1, 3], atol=1e-12)
+    assert np.allclose(st.dv[0, 0, 8, 0], [2, -2], atol=1e-12)
+    assert not st.dk[0, 0, :7].any() and not st.dk[0, 0, 9:].any()
+
+
+def test_context_keys_scale_free_values_linear(tiny_oracle):
+    """The context key is k-normed (invariant to the feature's scale); the value
+    is a plain projection (linear in it: no input norm)."""
+    o = tiny_oracle
+    f = np.random.default_rng(12).normal(size=(3, TINY.d))
+    s1, s2 = o.new_state(), o.new_state()
+    o.ctx_append(s1, 0, f, 20)
+    o.ctx_append(s2, 0, 3.0 * f, 20)
+    k1, k2 = s1.dk[:, 0, 20:23], s2.dk[:, 0, 20:23]
+    assert np.abs(k1 - k2).max() < 1e-4 * np.abs(k1).max()  # eps 1e-6 leaves about 1e-5
+    assert np.allclose(3.0 * s1.dv[:, 0, 20:23], s2.dv[:, 0, 20:23], atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
 # target forward: cached block forward == brute-force full recompute
 # ---------------------------------------------------------------------------
 
