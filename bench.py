@@ -48,6 +48,14 @@ def parse():
     p.add_argument("--profile-only", action="store_true", help="warmup + a few steps, no timing legs (for ncu)")
     p.add_argument("--depth", type=int, default=0,
                    help="with --profile-only: target layers of a reduced-depth copy (same widths), for small ncu captures")
+    # one projection through the tcgen05 GEMM alone (timing and ncu captures of that kernel)
+    p.add_argument("--kernel", choices=["gemm"], default=None,
+                   help="time one kernel instead of the round: gemm = out = X W^T with epilogue --mode")
+    p.add_argument("--N", type=int, default=151936)
+    p.add_argument("--K", type=int, default=4096)
+    p.add_argument("--M", type=int, default=17)
+    p.add_argument("--mode", type=int, default=4, help="0 fp32 store, 1 residual add, 2 SwiGLU, 3 SiLU, 4 argmax")
+    p.add_argument("--reps", type=int, default=3)
     return p.parse_args()
 
 
@@ -255,6 +263,51 @@ def run_reference(args):
 
 
 # --------------------------------------------------------------------------
+# one kernel alone: the tcgen05 projection (e.g. the LM head with its fused argmax)
+# --------------------------------------------------------------------------
+
+
+def run_kernel_gemm(args):
+    """`reps` launches of out = X W^T (bf16, N x K weights, M rows) with epilogue
+    `mode` through dflow_debug_gemm; CUDA-event time per launch and the achieved
+    algorithmic GB/s (weights + activations read once)."""
+    import torch
+
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    N, K, M, mode = args.N, args.K, args.M, args.mode
+    rows = max(64, ((M + 63) // 64) * 64)
+    cfg = synth.ModelConfig(name="gemm_kernel", dtype="bf16", d=128, n_layers=1, n_q_heads=1, n_kv_heads=1,
+                            head_dim=128, inter=64, vocab=max(N, 128), draft_layers=1, feat_layers=(1,), block=16,
+                            batch=rows // 64, prompt_len=64, new_tokens=16, schedule="uniform")
+    eng = Engine(cfg, random_weights(cfg), max_batch=cfg.batch, max_ctx=256)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    W = (torch.randn(N, K, generator=g, device="cuda") * 0.02).to(torch.bfloat16)
+    X = torch.randn(M, K, generator=g, device="cuda").to(torch.bfloat16)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    if mode in (0, 1):
+        out = torch.zeros(M, N, device="cuda")
+    elif mode in (2, 3):
+        out = torch.zeros(M, N // 2 if mode == 2 else N, dtype=torch.bfloat16, device="cuda")
+    else:
+        out = torch.zeros(M, dtype=torch.int32, device="cuda")
+    eng.debug_gemm(1, W, X, mode, out, st)  # warm-up (tensor maps, attributes)
+    torch.cuda.synchronize()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
+    evs[0].record()
+    for r in range(args.reps):
+        eng.debug_gemm(1, W, X, mode, out, st)
+        evs[r + 1].record()
+    torch.cuda.synchronize()
+    ms = [evs[r].elapsed_time(evs[r + 1]) for r in range(args.reps)]
+    alg = 2.0 * N * K + 2.0 * M * K
+    print(json.dumps({"kernel": "gemm", "N": N, "K": K, "M": M, "mode": mode, "status": int(st),
+                      "ms": [round(x, 4) for x in ms], "alg_bytes": alg,
+                      "gbs_best": round(alg / min(ms) / 1e6, 1)}), flush=True)
+
+
+# --------------------------------------------------------------------------
 # multi-GPU replicas: each rank runs its own batch; the step time is the slowest
 # rank's and the throughput the sum of all ranks' committed tokens
 # --------------------------------------------------------------------------
@@ -287,6 +340,8 @@ def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.kernel == "gemm":
+        return run_kernel_gemm(args)
     import torch
     import torch.distributed as dist
 

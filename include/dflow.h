@@ -68,7 +68,9 @@ enum { DFLOW_F32 = 0, DFLOW_BF16 = 1 };
 #define DFLOW_MAX_FEAT 8
 
 /* Model and workload shape.  head_dim must be 64 or 128, d_model a multiple
- * of 128, d_inter a multiple of 64.  feat_layers are 1-indexed target layers
+ * of 128, d_inter a multiple of 64.  DFLOW_BF16 runs on the tensor-core
+ * kernels: head_dim 128, page_size 64 and an sm_103 device (GB300; checked by
+ * dflow_set_workspace); DFLOW_F32 (a parity model) on CUDA cores.  feat_layers are 1-indexed target layers
  * (Eq. 1 takes the residual stream after each of them). */
 typedef struct dflow_config {
   int32_t dtype;
@@ -142,7 +144,8 @@ dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow
  * split-K / split-KV partials, the rotary table). */
 dflow_status dflow_workspace_size(const dflow_handle *h, size_t *bytes);
 /* Hand over scratch (>= dflow_workspace_size bytes, 256-byte aligned).  Fills
- * constant tables with a synchronous launch on the legacy default stream. */
+ * constant tables with a synchronous launch on the legacy default stream.
+ * DFLOW_ERR_UNSUPPORTED for a bf16 handle on a device other than sm_103. */
 dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes);
 dflow_status dflow_destroy(dflow_handle *h);
 
@@ -214,8 +217,10 @@ typedef struct dflow_kernel_profile {
 /* Turn per-launch event timing on (1) or off (0); either way clears the record. */
 dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable);
 /* Test hook: one projection out[m][n] = sum_k X[m][k] W[n][k] through the
- * library's GEMM kernels (path 0: CUDA-core kernel, path 1: tcgen05 kernel,
- * bf16 handles only), with the epilogue `mode`: 0 store fp32 out[M][ldo];
+ * library's GEMM kernels (path 0: CUDA-core kernel of fp32 handles; bf16
+ * handles: path 1 the tcgen05 kernel of one projection, path 2 the persistent
+ * tcgen05 launch the round uses for up to 128 rows (modes 0-3, K a multiple of
+ * 64 and at least 256); else DFLOW_ERR_UNSUPPORTED), with the epilogue `mode`: 0 store fp32 out[M][ldo];
  * 1 add into fp32 out[M][ldo]; 2 SwiGLU of 128-row [64 gate | 64 up] groups
  * into model-dtype out[M][ldo] (N/2 features); 3 SiLU into model-dtype out;
  * 4 greedy argmax over n into int32 out[M] (M <= max_batch * max(B+1, 64)).
@@ -235,13 +240,31 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
  *   tokens   int32 [rows]; all device pointers owned by the caller.
  * Limits: rows <= 64, vocab <= 262144 (else DFLOW_ERR_INVALID_ARG), d a
  * multiple of 64, sm_103 devices only (else DFLOW_ERR_UNSUPPORTED).
- * Scratch lives in a ~1 MiB array compiled into the library, held by every GPU
- * that loads it until exit.  The first call on a device looks up that array's
- * address (make it before any stream capture).  Calls share the array and it
- * keeps the last call's contents; calls that overlap on the GPU race.  Calls
- * no cudaMalloc/cudaFree and no allocating library routine. */
+ * Scratch lives in a ~1 MiB array compiled into the library.  It becomes
+ * device memory when the library's GPU code is loaded on a device (under
+ * CUDA's default lazy loading: at the first call there; CUDA_MODULE_LOADING=
+ * EAGER places it at library load) and is held until exit.  The first call on
+ * a device looks up the array's address (once per device, under a lock, so
+ * concurrent first calls are safe): make it at set-up, before any fixed-budget
+ * window or stream capture.  Calls share the array and it keeps the last
+ * call's contents; calls that overlap on the GPU race.  `stream` must belong to
+ * the current device (else DFLOW_ERR_INVALID_ARG).  Calls no cudaMalloc/
+ * cudaFree and no allocating library routine. */
 dflow_status dflow_greedy_tokens_noalloc(const void *lm_head, int32_t vocab, int32_t d, const void *hidden,
                                          int32_t rows, int32_t *tokens, void *stream);
+
+/* Test hook, host only (no GPU needed): the schedule the persistent tcgen05
+ * launch gives one GEMM of N x K weights over M rows on Q four-CTA clusters,
+ * computed by the functions the kernel itself evaluates.
+ *   plan  int32 [8]: padded columns, tiles T, k-blocks kb, full tiles Tf,
+ *         leftover tiles Tl, clusters per leftover tile ls, completion count of
+ *         the GEMM, leftover part slots available
+ *   ctas  int32 [Q*4][10], per CTA (cluster c/4, rank c%4): full tiles nt, first
+ *         tile t0, tile stride dt, k-block range [k0, k1), leftover tile lt (-1:
+ *         none), its k-block range [lk0, lk1), the cluster's part index, bytes
+ *         the CTA receives per split-K tile.
+ * DFLOW_ERR_UNSUPPORTED when M or K is outside what the launch covers. */
+dflow_status dflow_debug_seq_schedule(int32_t N, int32_t K, int32_t M, int32_t Q, int32_t *plan, int32_t *ctas);
 
 /* Waits for the recorded events, then fills out[DFLOW_PROF_N]. */
 dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out);

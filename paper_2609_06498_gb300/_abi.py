@@ -71,6 +71,8 @@ _SIGS = {
     "dflow_profile_read": ([_P, ctypes.POINTER(KernelProfile)], ctypes.c_int),
     "dflow_launch_count": ([_P, ctypes.POINTER(ctypes.c_uint64)], ctypes.c_int),
     "dflow_greedy_tokens_noalloc": ([_P, ctypes.c_int32, ctypes.c_int32, _P, ctypes.c_int32, _P, _P], ctypes.c_int),
+    "dflow_debug_seq_schedule": ([ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, c_i32p, c_i32p],
+                                 ctypes.c_int),
     "dflow_debug_gemm": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int32,
                           ctypes.c_int32, _P, ctypes.c_int32, _P, _P], ctypes.c_int),
 }

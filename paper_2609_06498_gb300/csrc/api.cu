@@ -572,19 +572,19 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
   const double es = h->esz;
   ProfScope ps(h, k.s, DFLOW_PROF_GEMM, es * N * K + es * M * K + ep_out_bytes(ep, M, N, h->esz), 2.0 * M * N * K);
   ++h->n_launch;
-  // few rows: the persistent kernel, one GEMM (all 36 clusters, balanced tiles)
-  static const bool single_tc = getenv("DFLOW_GEMM_TC_SINGLE") != nullptr;
+  if (!h->use_tc) {  // the fp32 parity model
+    h->dep.brk();
+    return gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, k.status, k.s);
+  }
+  // few rows: the persistent kernel, one GEMM (all clusters, balanced tiles)
   const bool seq_mode = ep.mode == EP_STORE_F32 || ep.mode == EP_RESID || ep.mode == EP_SWIGLU ||
                         ep.mode == EP_QKV || ep.mode == EP_SILU;
-  if (h->use_tc && !single_tc && seq_mode && h->dep.dev != nullptr && K % 64 == 0 && K / 64 >= 4 &&
-      ldx % 8 == 0 && seq_supported(M)) {
+  if (seq_mode && h->dep.dev != nullptr && K % 64 == 0 && K / 64 >= 4 && ldx % 8 == 0 && seq_supported(M)) {
     const SeqSpec sp{W, N, K, X, ldx, ep};
     return gemm_seq(h->tcw, 1, &sp, M, k.status_w, k.s, &h->dep);
   }
-  if (h->use_tc && tc_supports(N, K, M, ldx, ep))
-    return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
-  h->dep.brk();
-  return gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, k.status, k.s);
+  if (!tc_supports(N, K, M, ldx, ep)) return cudaErrorInvalidValue;
+  return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
 }
 
 EpArgs ep_f32(float *out, int ldo, int mode = EP_STORE_F32) {
@@ -1033,7 +1033,7 @@ dflow_status check_call(dflow_handle *h, const dflow_state *st) {
 
 // start of a call: its first counting launch waits for the previous grid; after a
 // failed call the counters are zeroed (a launch may have been counted but not run)
-Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
+void prep_chain(dflow_handle *h, void *stream) {
   DepChain &d = h->dep;
   if (d.dirty && d.dev != nullptr) {
     // with the counters, the persistent GEMM's leftover sums (a failed launch may have left partials)
@@ -1048,6 +1048,10 @@ Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
     }
   }
   d.brk();
+}
+
+Call make_call(dflow_handle *h, dflow_state *st, void *stream) {
+  prep_chain(h, stream);
   return Call{h, st->status, st->status, (cudaStream_t)stream};
 }
 
@@ -1092,6 +1096,7 @@ dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow
       c.max_ctx <= 0 || c.num_pages <= 0)
     return DFLOW_ERR_INVALID_ARG;
   if (c.head_dim != 64 && c.head_dim != 128) return DFLOW_ERR_UNSUPPORTED;
+  if (c.dtype == DFLOW_BF16 && (c.head_dim != 128 || c.page_size != 64)) return DFLOW_ERR_UNSUPPORTED;
   if (c.d_model % 128 || c.d_inter % 64 || c.n_q_heads % c.n_kv_heads || c.max_ctx % c.page_size)
     return DFLOW_ERR_UNSUPPORTED;
   if (c.n_feat < 1 || c.n_feat > DFLOW_MAX_FEAT) return DFLOW_ERR_INVALID_ARG;
@@ -1142,15 +1147,10 @@ dflow_status dflow_create(const dflow_config *cfg, const dflow_weights *w, dflow
   h->sm_count = sms > 0 ? sms : 148;
   const int sr = std::min(64, std::max(1, (2 * h->sm_count + c.n_kv_heads * c.max_batch - 1) / (c.n_kv_heads * c.max_batch)));
   h->attn_entries = std::max((size_t)h->rows_round * c.n_q_heads * sr, (size_t)h->rows_max * c.n_q_heads * std::min(sr, 4));
-  h->use_tc = false;
-  if (c.dtype == DFLOW_BF16) {
-    int major = 0, minor = 0;
-    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess &&
-        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess)
-      h->use_tc = (major == 10 && minor == 3) && getenv("DFLOW_DISABLE_TC") == nullptr;
-    cudaGetLastError();
-  }
-  h->fused = h->use_tc && c.head_dim == 128;
+  // bf16 models run on the tensor-core kernels (sm_103, checked when the
+  // workspace is handed over); fp32 (the parity model) on CUDA cores
+  h->use_tc = c.dtype == DFLOW_BF16;
+  h->fused = h->use_tc;
   h->ws_need = layout(h, nullptr);
   *out = h;
   return DFLOW_OK;
@@ -1164,6 +1164,16 @@ dflow_status dflow_workspace_size(const dflow_handle *h, size_t *bytes) {
 
 dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes) {
   if (!h || !dev || bytes < h->ws_need || ((uintptr_t)dev & 255)) return DFLOW_ERR_INVALID_ARG;
+  if (h->use_tc) {
+    int dev_id = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev_id) != cudaSuccess ||
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev_id) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev_id) != cudaSuccess) {
+      cudaGetLastError();
+      return DFLOW_ERR_CUDA;
+    }
+    if (major != 10 || minor != 3) return DFLOW_ERR_UNSUPPORTED;
+  }
   h->ws = static_cast<char *>(dev);
   h->ws_bytes = bytes;
   layout(h, h->ws);
@@ -1286,7 +1296,9 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
                               int32_t M, int32_t ldx, int32_t mode, void *out, int32_t ldo, int32_t *status,
                               void *stream) {
   if (!h || !h->ws || !W || !X || !out || !status || N < 1 || K < 1 || M < 1 || ldx < K) return DFLOW_ERR_INVALID_ARG;
-  if (path == 1 && (!h->use_tc || h->dtype != DFLOW_BF16)) return DFLOW_ERR_UNSUPPORTED;
+  if ((path >= 1) != (h->dtype == DFLOW_BF16) || path < 0 || path > 2) return DFLOW_ERR_UNSUPPORTED;
+  if (path == 2 && (mode == EP_ARGMAX || K % 64 || K / 64 < 4 || ldx % 8 || !seq_supported(M)))
+    return DFLOW_ERR_UNSUPPORTED;
   if (mode < 0 || mode > 4) return DFLOW_ERR_INVALID_ARG;
   if (mode == EP_ARGMAX && ((N + 127) / 128 > h->vocab_tiles || M > h->rows_max)) return DFLOW_ERR_INVALID_ARG;
   if (K % 32) return DFLOW_ERR_UNSUPPORTED;
@@ -1304,9 +1316,20 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
     ep.part_idx = h->am_idx;
     ep.n_tiles = (N + 127) / 128;
   }
-  cudaError_t e = (path == 1) ? (tc_supports(N, K, M, ldx, ep) ? gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, status, s)
-                                                              : cudaErrorNotSupported)
-                              : gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, status, s);
+  cudaError_t e;
+  if (path == 2) {
+    // the persistent launch the round uses for few-row projections, as one GEMM
+    prep_chain(h, stream);
+    if (h->dep.dev == nullptr) return DFLOW_ERR_UNSUPPORTED;
+    const SeqSpec sp{W, N, K, X, ldx, ep};
+    e = gemm_seq(h->tcw, 1, &sp, M, status, s, &h->dep);
+    h->dep.brk();
+    if (e != cudaSuccess) h->dep.dirty = true;
+  } else if (path == 1) {
+    e = tc_supports(N, K, M, ldx, ep) ? gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, status, s) : cudaErrorNotSupported;
+  } else {
+    e = gemm_simt(h->dtype, W, N, K, X, M, ldx, ep, status, s);
+  }
   if (e == cudaErrorNotSupported) return DFLOW_ERR_UNSUPPORTED;
   CK(e);
   if (mode == EP_ARGMAX) {

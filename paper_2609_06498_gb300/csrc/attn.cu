@@ -8,8 +8,6 @@
 // drafter's context positions 0..n-2 followed by the R block rows (no mask).
 // Each split writes an unnormalised partial (o, running max m, sum l); a
 // second kernel merges the splits.
-#include <stdlib.h>
-
 #include "dflow_internal.cuh"
 
 namespace dflow {
@@ -181,15 +179,11 @@ cudaError_t launch(const Dims &D, int batch, const AttnArgs &a, const int *statu
 
 cudaError_t attention(int dtype, const Dims &D, int batch, const AttnArgs &a, int *status, cudaStream_t s,
                       DepChain *chain) {
-  if (dtype == DFLOW_BF16 && attention_tc_supported(D) && getenv("DFLOW_SIMT_ATTENTION") == nullptr)
-    return attention_tc(D, batch, a, status, s, chain);
+  // bf16 caches: the tensor-core kernel; fp32 (the parity model): this one
+  if (dtype == DFLOW_BF16) return attention_tc(D, batch, a, status, s, chain);
   if (chain) chain->brk();
-  if (D.hd == 128)
-    return dtype == DFLOW_BF16 ? launch<bf16, 128>(D, batch, a, status, s)
-                               : launch<float, 128>(D, batch, a, status, s);
-  if (D.hd == 64)
-    return dtype == DFLOW_BF16 ? launch<bf16, 64>(D, batch, a, status, s)
-                               : launch<float, 64>(D, batch, a, status, s);
+  if (D.hd == 128) return launch<float, 128>(D, batch, a, status, s);
+  if (D.hd == 64) return launch<float, 64>(D, batch, a, status, s);
   return cudaErrorInvalidValue;
 }
 

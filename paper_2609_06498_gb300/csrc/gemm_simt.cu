@@ -1,5 +1,5 @@
-// CUDA-core GEMM with fused epilogues: the fp32 path (the fp32 parity config)
-// and the reference kernel the tensor-core GEMM is checked against.
+// CUDA-core GEMM with fused epilogues for the fp32 parity model (bf16 models
+// run every projection on the tensor-core kernels).
 //
 // out[m][n] = sum_k X[m][k] * W[n][k]; W row-major [N][K] (the layout of every
 // projection of the Qwen3 layer), X row-major [M][ldx].  A CTA computes a tile
@@ -111,9 +111,8 @@ cudaError_t launch(const void *W, int N, int K, const void *X, int M, int ldx, c
 cudaError_t gemm_simt(int dtype, const void *W, int N, int K, const void *X, int M, int ldx,
                       const EpArgs &ep, const int *status, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  if (K % TK != 0) return cudaErrorInvalidValue;
-  return dtype == DFLOW_BF16 ? launch<bf16>(W, N, K, X, M, ldx, ep, status, s)
-                             : launch<float>(W, N, K, X, M, ldx, ep, status, s);
+  if (K % TK != 0 || dtype != DFLOW_F32) return cudaErrorInvalidValue;
+  return launch<float>(W, N, K, X, M, ldx, ep, status, s);
 }
 
 }  // namespace dflow

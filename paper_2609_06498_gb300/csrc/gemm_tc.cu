@@ -387,9 +387,9 @@ __device__ __forceinline__ void st_async_f4(uint32_t caddr, const float4 &v, uin
                : "memory");
 }
 // split-K: token columns [s0, s1) of rank `rank` out of P (4-column groups)
-__device__ __forceinline__ int splitk_w4(int M, int P) { return ((M + 4 * P - 1) / (4 * P)) * 4; }
+__host__ __device__ __forceinline__ int splitk_w4(int M, int P) { return ((M + 4 * P - 1) / (4 * P)) * 4; }
 // bytes the owner of [s0, s1) receives per tile: a float4 per row and column group from each peer
-__device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
+__host__ __device__ __forceinline__ uint32_t splitk_recv_bytes(int P, int s0, int s1) {
   return s1 > s0 ? (uint32_t)((P - 1) * BM * ((s1 - s0 + 3) / 4) * 16) : 0u;
 }
 
@@ -871,8 +871,18 @@ struct SeqTab {
 __device__ __forceinline__ int sel4(const int (&a)[SEQ_MAX], int j) {
   return j == 0 ? a[0] : j == 1 ? a[1] : j == 2 ? a[2] : a[3];
 }
-// cta: this CTA's index in the grid (clusters are SEQ_P consecutive CTAs)
-__device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
+// high 32 bits of a 32 x 32-bit product (the schedule's divisions by runtime values)
+__host__ __device__ __forceinline__ unsigned int umulhi32(unsigned int a, unsigned int b) {
+#ifdef __CUDA_ARCH__
+  return __umulhi(a, b);
+#else
+  return (unsigned int)(((unsigned long long)a * b) >> 32);
+#endif
+}
+__host__ __device__ __forceinline__ int imin(int a, int b) { return a < b ? a : b; }
+// cta: this CTA's index in the grid (clusters are SEQ_P consecutive CTAs).  Also
+// evaluated on the host, where a test checks the schedule for every shape.
+__host__ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
   SeqTab t;
   t.n = p.n;
   const int q = cta / SEQ_P, rr = cta % SEQ_P;  // cluster, rank in the cluster
@@ -887,19 +897,19 @@ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) {
     t.k0[j] = rr * kb / SEQ_P;
     t.k1[j] = (rr + 1) * kb / SEQ_P;
     const bool left = on && q < g.Tl * g.ls;
-    const int lt = left ? (int)__umulhi((unsigned)q, g.ls_mag) : 0;
+    const int lt = left ? (int)umulhi32((unsigned)q, g.ls_mag) : 0;
     const int m = (q - lt * g.ls) * SEQ_P + rr;  // this CTA's part of its leftover tile
     t.lt[j] = left ? lt : -1;
     t.lpart[j] = left ? q - lt * g.ls : 0;
-    t.lk0[j] = left ? (int)__umulhi((unsigned)(m * kb), g.parts_mag) : 0;
-    t.lk1[j] = left ? (int)__umulhi((unsigned)((m + 1) * kb), g.parts_mag) : 0;
+    t.lk0[j] = left ? (int)umulhi32((unsigned)(m * kb), g.parts_mag) : 0;
+    t.lk1[j] = left ? (int)umulhi32((unsigned)((m + 1) * kb), g.parts_mag) : 0;
   }
   return t;
 }
 // bytes this CTA receives in a split-K tile of GEMM j
-__device__ __forceinline__ uint32_t seq_recv_bytes(int M, int npad, int rank) {
+__host__ __device__ __forceinline__ uint32_t seq_recv_bytes(int M, int npad, int rank) {
   const int w4 = npad / SEQ_P;
-  return splitk_recv_bytes(SEQ_P, min(rank * w4, M), min((rank + 1) * w4, M));
+  return splitk_recv_bytes(SEQ_P, imin(rank * w4, M), imin((rank + 1) * w4, M));
 }
 // true when this CTA has another tile after tile ti of GEMM j (ti = -1: its leftover part)
 __device__ __forceinline__ bool seq_more(const SeqTab &tb, int j, int ti) {
@@ -1506,10 +1516,30 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
   return cudaSuccess;
 }
 
-// leftover tiles split over several clusters (DFLOW_SEQ_NO_LEFTOVER: one cluster each)
-static bool seq_left_enabled() {
-  static const bool on = getenv("DFLOW_SEQ_NO_LEFTOVER") == nullptr;
-  return on;
+// The tile schedule of one GEMM of a persistent launch over Q clusters: T
+// tiles, of which the T mod Q left over from the round robin are split over
+// ls = Q / (T mod Q) clusters each, when that divides evenly, every part keeps a
+// k-block and the part slots exist (up to 64 columns: one epilogue chunk per
+// owner); cluster q then has nt_a + (q < nt_b) full tiles.
+static void seq_plan(SeqGemm &g, int N, int K, int M, int Q, int npad, bool have_slots) {
+  g.N = N;
+  g.K = K;
+  g.M = M;
+  g.T = (N + BM - 1) / BM;
+  g.kb = K / BK;
+  const int lo = g.T % Q;
+  g.Tf = g.T;
+  g.Tl = 0;
+  g.ls = 1;
+  if (lo > 0 && npad <= MAX_SPLIT_NPAD && Q <= SEQ_LEFT_MAX && Q % lo == 0 && g.kb >= SEQ_P * (Q / lo) && have_slots) {
+    g.Tf = g.T - lo;
+    g.Tl = lo;
+    g.ls = Q / lo;
+  }
+  g.nt_a = g.Tf / Q;
+  g.nt_b = g.Tf % Q;
+  g.ls_mag = g.ls > 1 ? (unsigned)((((uint64_t)1 << 32) + g.ls - 1) / g.ls) : 0u;
+  g.parts_mag = (unsigned)((((uint64_t)1 << 32) + SEQ_P * g.ls - 1) / (SEQ_P * g.ls));
 }
 
 // token columns of the persistent kernel for M rows: M rounded up to 16, and
@@ -1545,12 +1575,6 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   p.tmem_cols = cols;
   const size_t smem = seq_smem(p.npad, &p.stages, &p.rx_bytes);
   p.Q = seq_clusters(p.npad, smem);
-  // DFLOW_SEQ_CLUSTERS=n caps the grid at n clusters (all still resident at once)
-  static const int q_cap = [] {
-    const char *e = getenv("DFLOW_SEQ_CLUSTERS");
-    return e ? atoi(e) : 0;
-  }();
-  if (q_cap > 0 && q_cap < p.Q) p.Q = q_cap;
   if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
   const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   for (int j = 0; j < n; ++j) {
@@ -1563,30 +1587,12 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
          !(independent && sp[n - 1].ep.mode == EP_QKV && same_qkv_table(q.ep.qkv, sp[n - 1].ep.qkv))))
       return cudaErrorInvalidValue;
     SeqGemm &g = p.g[j];
-    g.N = q.N;
-    g.K = q.K;
-    g.M = M;
-    g.T = (q.N + BM - 1) / BM;
-    g.kb = q.K / BK;
     g.mode = mode;
-    // leftover tiles when they divide the clusters evenly and every part keeps a
-    // k-block (up to 64 columns: one epilogue chunk per owner)
-    const int lo = g.T % p.Q;
-    g.Tf = g.T;
-    g.Tl = 0;
-    g.ls = 1;
-    if (lo > 0 && p.npad <= MAX_SPLIT_NPAD && p.Q <= SEQ_LEFT_MAX && p.Q % lo == 0 && g.kb >= SEQ_P * (p.Q / lo) && w.lacc != nullptr &&
-        seq_left_enabled()) {
-      g.Tf = g.T - lo;
-      g.Tl = lo;
-      g.ls = p.Q / lo;
+    seq_plan(g, q.N, q.K, M, p.Q, p.npad, w.lacc != nullptr);
+    if (g.Tl > 0) {
       g.lacc = w.lacc + (size_t)j * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD;
       g.lctr = w.lctr + (size_t)j * SEQ_LEFT_MAX * SEQ_P;
     }
-    g.nt_a = g.Tf / p.Q;
-    g.nt_b = g.Tf % p.Q;
-    g.ls_mag = g.ls > 1 ? (unsigned)((((uint64_t)1 << 32) + g.ls - 1) / g.ls) : 0u;
-    g.parts_mag = (unsigned)((((uint64_t)1 << 32) + SEQ_P * g.ls - 1) / (SEQ_P * g.ls));
     g.idesc = idesc;
     g.ep = q.ep;
     g.ep.qkv.row0 = 0;
@@ -1632,3 +1638,29 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
 }
 
 }  // namespace dflow
+
+// Test hook (see include/dflow.h): the persistent launch's schedule of one GEMM
+// over Q clusters, computed by the same functions the kernel runs.
+extern "C" dflow_status dflow_debug_seq_schedule(int32_t N, int32_t K, int32_t M, int32_t Q, int32_t *plan,
+                                                 int32_t *ctas) {
+  using namespace dflow;
+  if (N < 1 || K < BK || K % BK || M < 1 || Q < 1 || Q > 1024 || !plan || !ctas) return DFLOW_ERR_INVALID_ARG;
+  const int npad = seq_npad(M);
+  if (npad > SEQ_MAX_NPAD || K / BK < SEQ_P) return DFLOW_ERR_UNSUPPORTED;
+  SeqParams p{};
+  p.n = 1;
+  p.M = M;
+  p.npad = npad;
+  p.Q = Q;
+  seq_plan(p.g[0], N, K, M, Q, npad, true);
+  const SeqGemm &g = p.g[0];
+  const int32_t pl[8] = {npad, g.T, g.kb, g.Tf, g.Tl, g.ls, SEQ_P * g.T, SEQ_LEFT_MAX};
+  for (int i = 0; i < 8; ++i) plan[i] = pl[i];
+  for (int c = 0; c < Q * SEQ_P; ++c) {
+    const SeqTab t = seq_tab(p, c);
+    const int32_t row[10] = {t.nt[0], t.t0[0], t.dt[0], t.k0[0], t.k1[0], t.lt[0], t.lk0[0], t.lk1[0], t.lpart[0],
+                             (int32_t)seq_recv_bytes(M, npad, c % SEQ_P)};
+    for (int i = 0; i < 10; ++i) ctas[(size_t)c * 10 + i] = row[i];
+  }
+  return DFLOW_OK;
+}

@@ -62,3 +62,15 @@ def token_check(got, ref_tokens, ref_logits, rows=None):
         elif got[i] != ref_tokens[i]:
             flips += 1
     return checked, flips
+
+
+def lmhead_engine(max_rows: int = 64):
+    """A bf16 handle whose workspace holds LM-head argmax partials for up to
+    max_rows rows over a 152064-token vocabulary (for GEMM-level tests)."""
+    import synth
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = synth.ModelConfig(name="lmhead", dtype="bf16", d=128, n_layers=1, n_q_heads=1, n_kv_heads=1, head_dim=128,
+                            inter=64, vocab=152064, draft_layers=1, feat_layers=(1,), block=16,
+                            batch=max_rows // 64 or 1, prompt_len=64, new_tokens=16, schedule="uniform")
+    return Engine(cfg, random_weights(cfg), max_batch=cfg.batch, max_ctx=256)
