@@ -45,6 +45,8 @@ def parse():
     p.add_argument("--relay", type=int, default=1, help="0 runs the DFlash baseline (no carry)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-other-workloads", action="store_true",
+                   help="skip the device legs of the other three bf16 workloads")
     p.add_argument("--profile-only", action="store_true", help="warmup + a few steps, no timing legs (for ncu)")
     p.add_argument("--depth", type=int, default=0,
                    help="with --profile-only: target layers of a reduced-depth copy (same widths), for small ncu captures")
@@ -161,14 +163,7 @@ class OracleSample:
         self.cfg = cfg
         self.vocab_div = vocab_div
         self.c1 = cfg.replace(n_layers=1, draft_layers=1, feat_layers=(1,), vocab=cfg.vocab // vocab_div)
-        block = np.random.default_rng(0).standard_normal(1 << 22, dtype=np.float32) * np.float32(0.02)
-        W = {}
-        for name, shape in synth.tensor_shapes(self.c1).items():
-            if len(shape) == 1:
-                W[name] = np.zeros(shape, np.float32) if name == "ln_b" else np.ones(shape, np.float32)
-            else:
-                W[name] = np.resize(block, int(np.prod(shape))).reshape(shape)
-        self.o = Oracle(self.c1, W)
+        self.o = Oracle(self.c1, timing_weights(self.c1))
         lens = synth.prompt_lengths(cfg) + 1
         self.st0 = self.o.state_from_synthetic(synth.synthetic_state(self.c1, ctx_lens=lens,
                                                                      n_carry=np.full(cfg.batch, cfg.block // 2)))
@@ -188,7 +183,7 @@ class OracleSample:
         setattr(self.o, name, w)
 
     def step(self, forced):
-        """One sampled round; returns (extrapolated full-round seconds, committed tokens)."""
+        """One sampled round: (measured seconds, extrapolated full-round seconds, committed tokens)."""
         st = self.st0.copy()
         self.acc = {}
         t0 = time.perf_counter()
@@ -201,56 +196,103 @@ class OracleSample:
         c = self.cfg
         full = (t + (c.n_layers - 1) * t_tlayer + (c.draft_layers - 1) * (t_dlayer + a.get("ctx_append", 0.0))
                 + (self.vocab_div - 1) * lm)
-        return full, int((ro.accept + 1).sum())
+        return t, full, int((ro.accept + 1).sum())
 
     def describe(self):
         c = self.cfg
         return (f"oracle round (numpy fp64) on a copy of {c.name} with 1 target + 1 draft layer and 1/"
                 f"{self.vocab_div} of the vocabulary (full width {c.d}, batch {c.batch}, context as the workload); "
-                f"time extrapolated to {c.n_layers}+{c.draft_layers} layers and the full LM head with timers on the "
-                f"oracle's own calls")
+                f"its measured time extrapolated to {c.n_layers}+{c.draft_layers} layers and the full LM head with "
+                f"timers on the oracle's own calls")
 
 
-# DRAM bytes (read + write) per algorithmic byte of the persistent layer-segment
-# GEMM launch, from one ncu capture of it at Qwen3-8B widths and 17 rows
-# (dram__bytes_read.sum + dram__bytes_write.sum = 390.7 MB for 387.3 MB of
-# weights, activations and outputs).  Valid for that kernel as captured.
-SEQ_TRAFFIC_RATIO = {"qwen3_8b_b1": 1.009}
+def timing_weights(cfg):
+    """Weights of the workload's shapes for timing the oracle: one random block
+    of N(0, 0.02) values reused for every matrix of the same name and shape
+    across layers and stacks (the oracle does the full arithmetic of every
+    layer; only the values repeat, which keeps host memory at one layer)."""
+    block = np.random.default_rng(0).standard_normal(1 << 22, dtype=np.float32) * np.float32(0.02)
+    shared, W = {}, {}
+    for name, shape in synth.tensor_shapes(cfg).items():
+        if len(shape) == 1:
+            W[name] = np.zeros(shape, np.float32) if name == "ln_b" else np.ones(shape, np.float32)
+            continue
+        base = name.split(".", 1)[1] if name[0] in "td" and name[1].isdigit() else name
+        key = (base, shape)
+        if key not in shared:
+            shared[key] = np.resize(block, int(np.prod(shape))).reshape(shape)
+        W[name] = shared[key]
+    return W
 
 
-def gemm_traffic(cfg, g):
-    """DRAM bytes of the mean GEMM launch of this run, scaled from the capture
-    (traffic grows with the weights streamed), or None without one."""
-    r = SEQ_TRAFFIC_RATIO.get(cfg.name)
-    if r is None or not g["launches"]:
-        return None
-    return round(r * g["bytes"] / g["launches"])
+def host_mem_available_gb() -> float:
+    try:
+        with open("/proc/meminfo") as f:
+            for ln in f:
+                if ln.startswith("MemAvailable:"):
+                    return int(ln.split()[1]) / 2 ** 20
+    except OSError:
+        pass
+    return 0.0
+
+
+def cpu_baseline_full_round(cfg, timed_sched):
+    """The oracle as it stands timed on one full-depth round of the workload
+    (every target and draft layer, full vocabulary, width, batch and context;
+    synthetic caches, layer-shared weight values), on this host's cores.
+    tokens/s = the schedule's mean committed tokens per round over the timed
+    rounds / the measured round time."""
+    from oracle import Oracle
+    mean_commit = float((np.asarray(timed_sched) + 1).sum(axis=1).mean())
+    if cfg.batch > 1 or host_mem_available_gb() < 48:
+        s = OracleSample(cfg)
+        tm, tf, _ = s.step(timed_sched[0])
+        return {"value": round(mean_commit / tf, 4), "unit": "tokens/s", "cores": s.threads, "kind": "oracle",
+                "sample": s.describe(), "sec_measured": round(tm, 2), "sec_per_round_est": round(tf, 2),
+                "mean_committed_per_round": mean_commit}
+    o = Oracle(cfg, timing_weights(cfg))
+    lens = synth.prompt_lengths(cfg) + 1
+    st = o.state_from_synthetic(synth.synthetic_state(cfg, ctx_lens=lens, n_carry=np.full(cfg.batch, cfg.block // 2)))
+    a = int(np.median(timed_sched))
+    t0 = time.perf_counter()
+    o.round(st, forced=[a] * cfg.batch)
+    sec = time.perf_counter() - t0
+    return {"value": round(mean_commit / sec, 4), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": (f"one full oracle round (numpy fp64) of {cfg.name}: {cfg.n_layers} target + "
+                       f"{cfg.draft_layers} draft layers, vocabulary {cfg.vocab}, width {cfg.d}, batch {cfg.batch}, "
+                       f"context {int(lens.max())} from a synthetic cache, forced a = {a}; weight values shared "
+                       f"across layers; tokens/s from the schedule's mean {mean_commit:.2f} committed per round"),
+            "sec_per_round": round(sec, 2), "mean_committed_per_round": mean_commit}
 
 
 def run_cpu_sample(cfg, steps: int, warmup: int, sched):
     s = OracleSample(cfg)
     for w in range(warmup):
         s.step(sched[w % len(sched)])
-    tot_t = tot_tok = 0.0
+    t_meas = t_full = tot_tok = 0.0
     for k in range(steps):
-        t, tok = s.step(sched[(warmup + k) % len(sched)])
-        tot_t += t
+        tm, tf, tok = s.step(sched[(warmup + k) % len(sched)])
+        t_meas += tm
+        t_full += tf
         tot_tok += tok
-    return tot_tok / tot_t, tot_t / steps, s
+    return tot_tok / t_full, t_meas / steps, t_full / steps, s
 
 
 def run_reference(args):
-    """Reference arm: the CPU oracle on a bounded sample of the workload."""
+    """Reference arm: the CPU oracle on a bounded sample of the workload.  A step
+    is one sampled round (measured: ms_per_step); the throughput is the sampled
+    rounds' committed tokens over their extrapolated full-round times."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     cfg = synth.CONFIGS[args.config]
     sched = synth.forced_schedule(cfg, args.warmup + args.steps)
     t0 = time.time()
-    value, sec_per_round, s = run_cpu_sample(cfg, args.steps, args.warmup, sched)
+    value, sec_meas, sec_full, s = run_cpu_sample(cfg, args.steps, args.warmup, sched)
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "tokens/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec_per_round * 1e3, 1),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec_meas * 1e3, 1),
+        "est_ms_per_full_round": round(sec_full * 1e3, 1),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": cfg.name, "batch": cfg.batch, "prompt": cfg.prompt_len, "block": cfg.block,
                    "l2": "inputs larger than L2"},
@@ -336,6 +378,93 @@ def replica_throughput(committed_local: float, ms_local: float, world: int, devi
 # --------------------------------------------------------------------------
 
 
+class Workload:
+    """A workload on the device: random-init weights, engine, prefilled state,
+    its forced acceptance schedule and `warmup` rounds already run; every leg
+    starts from the snapshot taken after them."""
+
+    def __init__(self, cfg, steps: int, warmup: int, rank: int = 0, relay: bool = True):
+        import torch
+
+        from paper_2609_06498_gb300 import Engine, random_weights
+        self.cfg, self.K, self.Wm = cfg, steps, warmup
+        n_rounds = warmup + steps
+        self.max_ctx = cfg.replace(new_tokens=n_rounds * cfg.rows).max_ctx()
+        self.weights = random_weights(cfg, seed=0)
+        self.eng = Engine(cfg, self.weights, max_batch=cfg.batch, max_ctx=self.max_ctx)
+        self.st = self.eng.new_state(cfg.batch, page_seed=rank)
+        self.eng.prefill(self.st, synth.prompts(cfg))
+        code = self.eng.read_status(self.st)
+        assert code == 0, f"prefill failed: device status {code}"
+        self.sched = synth.forced_schedule(cfg, n_rounds, seed=synth.SEED_SCHEDULE + rank)
+        self.forced = torch.as_tensor(self.sched).cuda()
+        self.acc = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
+        self.comm = torch.empty(cfg.batch, cfg.rows, dtype=torch.int32, device="cuda")
+        for w in range(warmup):
+            self.round(w, relay)
+        torch.cuda.synchronize()
+        self.snap = {k: getattr(self.st, k).clone() for k in ("tokens", "seq_len", "carry", "n_carry", "boundary")}
+        # a+1 committed per sequence per round (forced a) over the timed rounds
+        self.committed = float((self.sched[warmup:n_rounds] + 1).sum())
+        ctx0 = float(self.snap["seq_len"].float().mean())
+        self.mean_ctx = ctx0 + float((self.sched[warmup:n_rounds] + 1).mean()) * steps / 2
+
+    def round(self, r: int, relay: bool = True):
+        self.eng.round(self.st, self.forced[r], relay=relay, out=(self.acc, self.comm))
+
+    def restore(self):
+        import torch
+        for k, v in self.snap.items():
+            getattr(self.st, k).copy_(v)
+        torch.cuda.synchronize()
+
+    def device_leg(self, relay: bool = True, barrier=None):
+        """K rounds back to back from the snapshot: per-round CUDA-event times
+        (ms) on the launching stream, the total, and the library's launches."""
+        import torch
+        self.restore()
+        stream = torch.cuda.current_stream()
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(self.K + 1)]
+        n0 = self.eng.launch_count()
+        if barrier:
+            barrier()
+        ev[0].record(stream)
+        for k in range(self.K):
+            self.round(self.Wm + k, relay)
+            ev[k + 1].record(stream)
+        torch.cuda.synchronize()
+        launches = self.eng.launch_count() - n0
+        code = self.eng.read_status(self.st)
+        assert code == 0, f"device status {code} set during the timed leg"
+        per = [ev[k].elapsed_time(ev[k + 1]) for k in range(self.K)]
+        return per, ev[0].elapsed_time(ev[self.K]), launches
+
+    def release(self):
+        import torch
+        for k in ("eng", "st", "weights", "forced", "snap"):
+            setattr(self, k, None)
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+
+
+def round_summary(cfg, per, total_ms, committed, mean_ctx):
+    """ms per round, committed tokens/s and the round's HBM roofline fraction."""
+    hbm, _, peak_src = peaks()
+    K = len(per)
+    ms = total_ms / K
+    rb = round_bytes(cfg, mean_ctx)
+    gbs = rb["total"] / (ms / 1e3) / 1e9
+    return {"ms_per_round": round(ms, 4), "p50_ms": round(float(np.percentile(per, 50)), 4),
+            "tokens_per_s": round(committed / (total_ms / 1e3), 2), "batch": cfg.batch,
+            "acceptance": f"forced {cfg.schedule}", "rounds": K,
+            "round_roofline": {"alg_bytes": rb["total"], "achieved_gbs": round(gbs, 1), "peak": hbm,
+                               "frac": round(gbs / hbm, 4), "peak_source": peak_src}}
+
+
+# the other bf16 workloads measured in the default run (device leg only)
+OTHER_WORKLOADS = ("qwen3_1p7b_b1", "qwen3_4b_b4", "qwen3_8b_kv_b16")
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -345,7 +474,7 @@ def main():
     import torch
     import torch.distributed as dist
 
-    from paper_2609_06498_gb300 import Engine, build, random_weights
+    from paper_2609_06498_gb300 import build
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -365,31 +494,9 @@ def main():
                           feat_layers=tuple(sorted({1, args.depth})))
     K, Wm = args.steps, args.warmup
     relay = bool(args.relay)  # 0: the DFlash baseline (mask embeddings only, nothing carried)
-    n_rounds = Wm + K
     lens = synth.prompt_lengths(cfg)
-    max_ctx = cfg.replace(new_tokens=n_rounds * cfg.rows).max_ctx()
-    weights = random_weights(cfg, seed=0)
-    eng = Engine(cfg, weights, max_batch=cfg.batch, max_ctx=max_ctx)
-    st = eng.new_state(cfg.batch, page_seed=rank)
-    prompts = synth.prompts(cfg)
-    eng.prefill(st, prompts)
-    st_code = eng.read_status(st)
-    assert st_code == 0, f"prefill failed: device status {st_code}"
-    sched = synth.forced_schedule(cfg, n_rounds, seed=synth.SEED_SCHEDULE + rank)
-    forced_dev = torch.as_tensor(sched).cuda()
-    acc = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
-    comm = torch.empty(cfg.batch, cfg.rows, dtype=torch.int32, device="cuda")
-
-    for w in range(Wm):
-        eng.round(st, forced_dev[w], relay=relay, out=(acc, comm))
-    torch.cuda.synchronize()
-    # snapshot of the per-sequence state after warmup: every leg starts from it
-    snap = {k: getattr(st, k).clone() for k in ("tokens", "seq_len", "carry", "n_carry", "boundary")}
-
-    def restore():
-        for k, v in snap.items():
-            getattr(st, k).copy_(v)
-        torch.cuda.synchronize()
+    wl = Workload(cfg, K, Wm, rank, relay)
+    eng, st = wl.eng, wl.st
 
     def barrier():
         if world > 1:
@@ -400,38 +507,24 @@ def main():
         # rounds inside a profiler range, for `ncu --profile-from-start off`
         torch.cuda.cudart().cudaProfilerStart()
         for k in range(min(K, 2)):
-            eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
+            wl.round(Wm + k, relay)
         torch.cuda.synchronize()
         torch.cuda.cudart().cudaProfilerStop()
         print(json.dumps({"profile_only": True, "launches": eng.launch_count()}))
         return
 
-    committed = float((sched[Wm:Wm + K] + 1).sum())  # a+1 per sequence per round (forced a)
-    ctx0 = float(snap["seq_len"].float().mean())
-    mean_ctx = ctx0 + float((sched[Wm:Wm + K] + 1).mean()) * K / 2
+    committed, mean_ctx, sched = wl.committed, wl.mean_ctx, wl.sched
+    stream = torch.cuda.current_stream()
 
     # ---- device leg: K rounds back to back, CUDA events on the launching stream
-    restore()
-    stream = torch.cuda.current_stream()
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
-    n0 = eng.launch_count()
     with ClockSampler(local) as clocks:
-        barrier()
-        ev[0].record(stream)
-        for k in range(K):
-            eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
-            ev[k + 1].record(stream)
-        torch.cuda.synchronize()
-    launches = eng.launch_count() - n0
-    st_code = eng.read_status(st)
-    assert st_code == 0, f"device status {st_code} set during the timed leg"
-    per = [ev[k].elapsed_time(ev[k + 1]) for k in range(K)]
-    value, total_ms = replica_throughput(committed, ev[0].elapsed_time(ev[K]), world, "cuda")
+        per, total_local, launches = wl.device_leg(relay, barrier)
+    value, total_ms = replica_throughput(committed, total_local, world, "cuda")
 
     # ---- end-to-end leg: host buffers, H2D of the step's inputs and D2H of its result inside the region
     e2e = None
     if not args.no_e2e:
-        restore()
+        wl.restore()
         h_forced = torch.as_tensor(sched).pin_memory()
         h_acc = torch.empty(K, cfg.batch, dtype=torch.int32).pin_memory()
         h_comm = torch.empty(K, cfg.batch, cfg.rows, dtype=torch.int32).pin_memory()
@@ -441,9 +534,9 @@ def main():
         e0.record(stream)
         for k in range(K):
             d_forced.copy_(h_forced[Wm + k], non_blocking=True)
-            eng.round(st, d_forced, relay=relay, out=(acc, comm))
-            h_acc[k].copy_(acc, non_blocking=True)
-            h_comm[k].copy_(comm, non_blocking=True)
+            eng.round(st, d_forced, relay=relay, out=(wl.acc, wl.comm))
+            h_acc[k].copy_(wl.acc, non_blocking=True)
+            h_comm[k].copy_(wl.comm, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_value, _ = replica_throughput(committed, e0.elapsed_time(e1), world, "cuda")
@@ -453,7 +546,7 @@ def main():
 
     # ---- per-step split: the round's four calls one at a time, events between them
     # (the per-call entry points draft and carry with the relay on)
-    restore()
+    wl.restore()
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
     for k in range(K):
         e = evs[k]
@@ -462,7 +555,7 @@ def main():
         e[1].record(stream)
         g_t, feats, _ = eng.verify_block(st, blk)
         e[2].record(stream)
-        a_k, _ = eng.accept_commit(st, blk, g_t, forced_dev[Wm + k])
+        a_k, _ = eng.accept_commit(st, blk, g_t, wl.forced[Wm + k])
         e[3].record(stream)
         eng.carry_hidden(st, blk, feats, a_k)
         e[4].record(stream)
@@ -472,11 +565,20 @@ def main():
     step_split = {name: round(float(np.median([evs[k][i].elapsed_time(evs[k][i + 1]) for k in range(K)])), 4)
                   for i, name in enumerate(("draft", "verify", "accept", "carry"))}
 
+    # ---- relay off (the DFlash baseline of Sec. 5.3's runtime-overhead figure): same state and schedule
+    relay_cost = None
+    if rank == 0 and world == 1 and relay:
+        per_off, total_off, _ = wl.device_leg(False)
+        on, off = total_local / K, total_off / K
+        relay_cost = {"dflow_ms": round(on, 4), "dflash_ms": round(off, 4), "delta_ms": round(on - off, 4),
+                      "delta_frac": round((on - off) / off, 4),
+                      "paper": "0.51 ms, 1.2 % of a DFlash round (Sec. 5.3; A800, model not stated)"}
+
     # ---- profiled leg: per-launch events around the GEMMs (the dominant kernel)
-    restore()
+    wl.restore()
     eng.profile(True)
     for k in range(K):
-        eng.round(st, forced_dev[Wm + k], relay=relay, out=(acc, comm))
+        wl.round(Wm + k, relay)
     torch.cuda.synchronize()
     prof = eng.profile_read()
     eng.profile(False)
@@ -507,14 +609,26 @@ def main():
                            "frac": round(round_gbs / hbm, 4), "unit": "GB/s", "peak_source": peak_src},
         "phase_ms": {"gemm": round(g["ms"] / K, 4), "attention": round(prof["attn"]["ms"] / K, 4)},
         "step_split_ms": step_split,
+        "relay_overhead": relay_cost,
         "gpu_launches": int(launches),
         "e2e": e2e,
         "clocks": clocks.summary(),
     }
+    wl.release()
+
+    # ---- the other workloads (device leg, rank 0, one GPU): min(K, 20) rounds after min(W, 5)
+    if rank == 0 and world == 1 and not args.no_other_workloads and cfg.name == DEFAULT_CONFIG:
+        others = {}
+        for name in OTHER_WORKLOADS:
+            c = synth.CONFIGS[name]
+            w = Workload(c, min(K, 20), min(Wm, 5))
+            per_o, tot_o, _ = w.device_leg()
+            others[name] = round_summary(c, per_o, tot_o, w.committed, w.mean_ctx)
+            w.release()
+        line["workloads"] = others
+
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cv, cs, s = run_cpu_sample(cfg, steps=1, warmup=0, sched=sched)
-        line["cpu_baseline"] = {"value": round(cv, 4), "unit": "tokens/s", "cores": s.threads, "kind": "oracle",
-                                "sample": s.describe(), "sec_per_round": round(cs, 2)}
+        line["cpu_baseline"] = cpu_baseline_full_round(cfg, sched[Wm:Wm + K])
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -160,8 +160,10 @@ dflow_status dflow_prefill(dflow_handle *h, dflow_state *st, const int32_t *prom
 
 /* Sec. 3 Eq. 2 + Sec. 4.2 Eq. 4-5.  block_tokens int32 [batch][B+1]: row 0 =
  * anchor, rows 1..B = drafter argmax.  Reads tokens, seq_len, drafter
- * context, carry, n_carry, boundary. */
-dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens,
+ * context, carry, n_carry, boundary.  If logits is non-null, also the
+ * drafter's fp32 logits [batch][B+1][vocab] (row 0 included; a second pass
+ * over the LM head, for tests). */
+dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens, float *logits,
                                void *stream);
 
 /* Sec. 3 Eq. 3 (target forward) + Eq. 1.  Reads block_tokens [batch][B+1];

@@ -61,7 +61,7 @@ _SIGS = {
     "dflow_set_workspace": ([_P, _P, ctypes.c_size_t], ctypes.c_int),
     "dflow_destroy": ([_P], ctypes.c_int),
     "dflow_prefill": ([_P, ctypes.POINTER(State), _P, ctypes.c_int32, c_i32p, _P], ctypes.c_int),
-    "dflow_draft_block": ([_P, ctypes.POINTER(State), _P, _P], ctypes.c_int),
+    "dflow_draft_block": ([_P, ctypes.POINTER(State), _P, _P, _P], ctypes.c_int),
     "dflow_verify_block": ([_P, ctypes.POINTER(State), _P, _P, _P, _P, _P], ctypes.c_int),
     "dflow_accept_commit": ([_P, ctypes.POINTER(State), _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dflow_carry_hidden": ([_P, ctypes.POINTER(State), _P, _P, _P, _P], ctypes.c_int),

@@ -902,7 +902,7 @@ Dims round_dims(const dflow_handle *h) {
 }
 
 template <typename T>
-dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
+dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float *logits = nullptr) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R, B = D.B;
@@ -937,7 +937,7 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay) {
   const int splits = pick_splits(h, batch, rows);
   CK(stack_forward<T>(k, D, batch, h->dl.data(), h->cfg.draft_layers, static_cast<T *>(st->draft_kv), st, 0, splits,
                       h->w.draft_final_norm));
-  CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, nullptr));
+  CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, logits));
   KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
                                                    D.R, blk, k.status));
   CK(cudaGetLastError());
@@ -1208,14 +1208,15 @@ dflow_status dflow_prefill(dflow_handle *h, dflow_state *st, const int32_t *prom
                                           : do_prefill<float>(k, st, prompt, prompt_stride, prompt_len_host));
 }
 
-dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens, void *stream) {
+dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_tokens, float *logits,
+                               void *stream) {
   dflow_status r = check_call(h, st);
   if (r) return r;
   if (!block_tokens) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
   if ((r = guard(k, st))) return finish(h, r);
-  return finish(h, h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1)
-                                          : do_draft<float>(k, st, block_tokens, 1));
+  return finish(h, h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1, logits)
+                                          : do_draft<float>(k, st, block_tokens, 1, logits));
 }
 
 dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t *block_tokens,

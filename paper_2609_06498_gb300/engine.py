@@ -221,10 +221,14 @@ class Engine:
              lens.ctypes.data_as(_abi.c_i32p), self._stream())
         torch.cuda.current_stream().synchronize()
 
-    def draft_block(self, st: DeviceState) -> torch.Tensor:
+    def draft_block(self, st: DeviceState, logits: bool = False):
+        """Block tokens [batch][B+1]; with logits=True also the drafter's fp32 logits."""
         blk = self._i32(st.batch, self.cfg.rows)
-        call("dflow_draft_block", self.h, ctypes.byref(st.c), ctypes.c_void_p(blk.data_ptr()), self._stream())
-        return blk
+        lg = (torch.empty(st.batch, self.cfg.rows, self.cfg.vocab, dtype=torch.float32, device=self.device)
+              if logits else None)
+        call("dflow_draft_block", self.h, ctypes.byref(st.c), ctypes.c_void_p(blk.data_ptr()),
+             ctypes.c_void_p(lg.data_ptr() if lg is not None else 0), self._stream())
+        return (blk, lg) if logits else blk
 
     def verify_block(self, st: DeviceState, blk: torch.Tensor, logits: bool = False):
         g = self._i32(st.batch, self.cfg.rows)

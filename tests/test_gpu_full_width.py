@@ -17,18 +17,21 @@ from parity_util import assert_close, to_np, token_check, upload_state
 
 pytestmark = pytest.mark.gpu
 
-FULL = [synth.QWEN3_1P7B, synth.QWEN3_4B, synth.QWEN3_8B, synth.QWEN3_8B_KV]
-
-
 def reduced(cfg):
     return cfg.replace(n_layers=2, draft_layers=1, feat_layers=(1, 2))
+
+
+# the four bf16 workloads at 2 + 1 layers, and the headline workload with its
+# five feature layers (Eq. 1 over m = 5 layers: W_c is 4096 x 20480)
+FULL = [reduced(synth.QWEN3_1P7B), reduced(synth.QWEN3_4B), reduced(synth.QWEN3_8B), reduced(synth.QWEN3_8B_KV),
+        synth.QWEN3_8B.replace(name="qwen3_8b_b1_m5", n_layers=5, draft_layers=1, feat_layers=(1, 2, 3, 4, 5))]
 
 
 @pytest.fixture(scope="module", params=FULL, ids=lambda c: c.name)
 def full(request):
     from paper_2609_06498_gb300 import Engine, build, pack_weights
     build.build()
-    cfg = reduced(request.param)
+    cfg = request.param
     W = synth.weights(cfg, perturb_norms=True)
     eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
     o = Oracle(cfg, {k: v.astype(np.float64) for k, v in W.items()})
@@ -47,13 +50,15 @@ def test_full_width_round_calls(full):
     upload_state(eng, st, ost)
     ref = ost.copy()
 
-    # draft (Eq. 2, Eq. 4-5)
-    gblk = to_np(eng.draft_block(st))
+    # draft (Eq. 2, Eq. 4-5): logits elementwise, tokens where the decision is safe
+    gblk, gdl = eng.draft_block(st, logits=True)
+    gblk, gdl = to_np(gblk), to_np(gdl)
     oblk = np.zeros((bs, R), np.int32)
     checked = 0
     for b in range(bs):
         oblk[b], lg, _ = o.draft_block(ref, b)
         assert gblk[b, 0] == oblk[b, 0]
+        assert_close(gdl[b, 1:], lg[1:], cfg, "draft logits")
         c, _ = token_check(gblk[b], oblk[b], lg, rows=range(1, R))
         checked += c
     assert checked >= bs * (B // 2)
@@ -102,6 +107,48 @@ def test_full_width_round_calls(full):
         assert_close(to_np(dk)[:, lo:], ref.dk[:, b, lo:n - 1], cfg, "ctx K append")
         assert_close(to_np(dv)[:, lo:], ref.dv[:, b, lo:n - 1], cfg, "ctx V append")
     assert eng.read_status(st) == 0
+
+
+@pytest.mark.parametrize("name", ["qwen3_8b_b1", "qwen3_4b_b4"])
+def test_full_width_rounds(name):
+    """Three dflow_round calls in a row at full widths (2 + 1 layers) from a
+    synthetic state, against the oracle's rounds: acceptance, commits, lengths,
+    carry counts and boundaries bit exact, carried states at tolerance.  Each
+    round starts from the oracle's state (resynchronised after an allowed
+    near-tie flip), as in the small-model round test."""
+    from oracle import top2_gap
+    from paper_2609_06498_gb300 import Engine, build, pack_weights
+    build.build()
+    cfg = reduced(synth.CONFIGS[name])
+    W = synth.weights(cfg, perturb_norms=True)
+    eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
+    o = Oracle(cfg, {k: v.astype(np.float64) for k, v in W.items()})
+    lens = synth.prompt_lengths(cfg) + 1
+    nc = np.array([[5, 0, 15, 9][b % 4] for b in range(cfg.batch)], np.int32)
+    ost = o.state_from_synthetic(synth.synthetic_state(cfg, ctx_lens=lens, n_carry=nc))
+    st = eng.new_state(cfg.batch, page_seed=17)
+    sched = synth.forced_schedule(cfg, 3)
+    exact = 0
+    for r in range(3):
+        upload_state(eng, st, ost)
+        acc, comm = eng.round(st, torch.as_tensor(sched[r]).cuda())
+        ro = o.round(ost, forced=list(sched[r]))
+        assert eng.read_status(st) == 0
+        ga, gc = to_np(acc), to_np(comm)
+        assert np.array_equal(ga, ro.accept)  # forced
+        for b in range(cfg.batch):
+            if np.array_equal(gc[b], ro.committed[b]):
+                exact += 1
+                assert int(st.seq_len[b]) == int(ost.seq_len[b])
+                assert int(st.n_carry[b]) == int(ost.n_carry[b])
+                nc_b = int(ost.n_carry[b])
+                if nc_b:
+                    assert_close(to_np(st.carry)[b, :nc_b], ost.carry[b, :nc_b], cfg, "carried states")
+                assert int(to_np(st.boundary)[b, 0]) == int(ost.boundary[b, 0])
+            else:
+                gaps = np.concatenate([top2_gap(ro.draft_logits[b][1:]), top2_gap(ro.verify_logits[b])])
+                assert gaps.min() <= 0.05, f"round {r} seq {b}: diverged without a near tie"
+    assert exact >= 2 * cfg.batch
 
 
 def test_full_depth_8b_round_invariants():

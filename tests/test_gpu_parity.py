@@ -88,15 +88,18 @@ def test_per_call_parity(setup):
     ref = ost.copy()
     R, B = cfg.rows, cfg.block
 
-    # dflow_draft_block (Eq. 2, Eq. 4-5)
-    blk = eng.draft_block(st)
-    gblk = to_np(blk)
+    # dflow_draft_block (Eq. 2, Eq. 4-5): drafter logits elementwise, tokens where safe
+    blk, dlogits = eng.draft_block(st, logits=True)
+    gblk, gdl = to_np(blk), to_np(dlogits)
     oblk = np.zeros((cfg.batch, R), np.int32)
+    checked = 0
     for b in range(cfg.batch):
         oblk[b], lg, _ = o.draft_block(ref, b)
         assert gblk[b, 0] == oblk[b, 0]
-        checked, _ = token_check(gblk[b], oblk[b], lg, rows=range(1, R))
-        assert checked >= 1
+        assert_close(gdl[b, 1:], lg[1:], cfg, "draft logits")
+        c, _ = token_check(gblk[b], oblk[b], lg, rows=range(1, R))
+        checked += c
+    assert checked >= cfg.batch * (R - 1) // 4
 
     # dflow_verify_block (Eq. 3 target side, Eq. 1) on the oracle's block
     blk_t = torch.as_tensor(oblk).cuda()
@@ -157,9 +160,12 @@ def test_per_call_parity(setup):
     assert eng.read_status(st) == 0
 
 
-def test_round_parity(setup):
+@pytest.mark.parametrize("relay", [True, False], ids=["dflow", "relay_off"])
+def test_round_parity(setup, relay):
     """dflow_round from the oracle's state, several rounds, resynchronised from
-    the oracle whenever an allowed near-tie flip makes the two diverge."""
+    the oracle whenever an allowed near-tie flip makes the two diverge.  relay
+    off is the DFlash baseline of Sec. 5.3 (mask embeddings only, nothing
+    carried: Eq. 5 with no valid slot)."""
     cfg, W, o, eng = setup
     ost = _oracle_round_state(cfg, o)
     st = eng.new_state(cfg.batch, page_seed=11)
@@ -168,8 +174,8 @@ def test_round_parity(setup):
     for r in range(6):
         upload_state(eng, st, ost)
         forced = sched[r] if cfg.schedule != "natural" else None
-        acc, comm = eng.round(st, torch.as_tensor(forced).cuda() if forced is not None else None)
-        ro = o.round(ost, forced=None if forced is None else list(forced))
+        acc, comm = eng.round(st, torch.as_tensor(forced).cuda() if forced is not None else None, relay=relay)
+        ro = o.round(ost, forced=None if forced is None else list(forced), relay=relay)
         assert eng.read_status(st) == 0
         ga, gc = to_np(acc), to_np(comm)
         for b in range(cfg.batch):
@@ -177,6 +183,8 @@ def test_round_parity(setup):
                 exact_rounds += 1
                 assert int(st.seq_len[b]) == int(ost.seq_len[b])
                 assert int(st.n_carry[b]) == int(ost.n_carry[b])
+                if not relay:
+                    assert int(st.n_carry[b]) == 0
                 gb = to_np(st.boundary)[b]
                 assert gb[0] == ost.boundary[b, 0]
                 a = int(ro.accept[b])
@@ -202,7 +210,7 @@ def test_round_parity_separate_gemms(setup, monkeypatch):
     if cfg.dtype != "bf16" or cfg.head_dim != 128:
         pytest.skip("the persistent GEMM sequence is the bf16 path with 128-dim heads")
     monkeypatch.setenv("DFLOW_SEPARATE_GEMMS", "1")
-    test_round_parity(setup)
+    test_round_parity(setup, True)
 
 
 def test_generate_matches_oracle_tiny():
@@ -251,9 +259,11 @@ def test_long_context_per_call(ctx):
     eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
     st = eng.new_state(cfg.batch, page_seed=5)
     upload_state(eng, st, ost)
-    blk = to_np(eng.draft_block(st))
+    blk, dl = eng.draft_block(st, logits=True)
+    blk, dl = to_np(blk), to_np(dl)
     for b in range(cfg.batch):
         oblk, lg, _ = o.draft_block(ost, b)
+        assert_close(dl[b, 1:], lg[1:], cfg, "draft logits")
         token_check(blk[b], oblk, lg, rows=range(1, cfg.rows))
     oblk = synth.block_tokens(cfg, ost.tokens[np.arange(cfg.batch), ost.seq_len - 1])
     g, feats, logits = eng.verify_block(st, torch.as_tensor(oblk).cuda(), logits=True)
