@@ -198,6 +198,18 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
                          int32_t *accept_len, int32_t *committed, int32_t relay,
                          void *stream);
 
+/* Sec. 5.2, Table 2 "Baseline": one step of plain autoregressive greedy
+ * decoding of the target, for every active sequence: the last committed token
+ * (position n-1) runs through the target against the cached K/V (its K/V are
+ * written), and its greedy prediction is committed: tokens[n], seq_len = n+1.
+ * token_out int32 [batch] (-1 for inactive sequences).  Afterwards nothing is
+ * carried (n_carry = 0, boundary = -1).  draft_context = 1 also appends the
+ * row's Eq. 1 feature to the drafter context, so dflow_round may follow; with
+ * 0 (the plain baseline) the drafter context falls behind and no round should
+ * follow on that state. */
+dflow_status dflow_decode_step(dflow_handle *h, dflow_state *st, int32_t *token_out, int32_t draft_context,
+                               void *stream);
+
 /* Synchronises `stream`, then copies *state->status to *host_status. */
 dflow_status dflow_read_status(dflow_handle *h, const dflow_state *st, int32_t *host_status,
                                void *stream);

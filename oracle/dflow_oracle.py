@@ -16,6 +16,7 @@ in the order the paper states the method:
   * Sec. 4.2, Eq. 4 -- reject-conditioned MLP  [beta; gamma] = MLP([E(b); E(y_{a+1}); h])
   * Sec. 4.2, Eq. 5 -- x = E_mask + beta * LN(h) + gamma at valid carried slots,
                       E_mask elsewhere, masks only when nothing is carried
+  * Sec. 5.2        -- the autoregressive baseline (one greedy target step)
 
 Readings of points the paper leaves open (all shared with the CUDA path by
 specification, not by code):
@@ -442,6 +443,25 @@ class Oracle:
                 rounds_out.append(ro)
             r += 1
         return [st.tokens[b, plen[b]:plen[b] + n_new].copy() for b in range(self.cfg.batch)], st
+
+    # -- plain autoregressive decoding (Sec. 5.2, Table 2 "Baseline") ----------
+
+    def decode_step(self, st: State, b: int, draft_context: bool = False):
+        """One step of ordinary greedy decoding of the target with its KV cache:
+        the last committed token (position n-1) runs through the target, its
+        K/V join the cache, and its greedy prediction is committed (n grows by
+        one).  draft_context: the row's Eq. 1 feature also joins the drafter
+        context, so that speculative rounds can follow.  Returns the token."""
+        n = int(st.seq_len[b])
+        logits, feats = self.target_forward(st, b, [int(st.tokens[b, n - 1])], n - 1)
+        tok = int(argmax_rows(logits)[0])
+        st.tokens[b, n] = tok
+        st.seq_len[b] = n + 1
+        if draft_context:
+            self.ctx_append(st, b, feats, n - 1)
+        st.n_carry[b] = 0
+        st.boundary[b] = -1
+        return tok, logits[0]
 
     # -- brute-force greedy reference (no cache, full causal recompute) -------
 

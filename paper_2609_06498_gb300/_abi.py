@@ -65,6 +65,7 @@ _SIGS = {
     "dflow_verify_block": ([_P, ctypes.POINTER(State), _P, _P, _P, _P, _P], ctypes.c_int),
     "dflow_accept_commit": ([_P, ctypes.POINTER(State), _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dflow_carry_hidden": ([_P, ctypes.POINTER(State), _P, _P, _P, _P], ctypes.c_int),
+    "dflow_decode_step": ([_P, ctypes.POINTER(State), _P, ctypes.c_int32, _P], ctypes.c_int),
     "dflow_round": ([_P, ctypes.POINTER(State), _P, _P, _P, ctypes.c_int32, _P], ctypes.c_int),
     "dflow_read_status": ([_P, ctypes.POINTER(State), c_i32p, _P], ctypes.c_int),
     "dflow_profile_enable": ([_P, ctypes.c_int32], ctypes.c_int),

@@ -79,6 +79,33 @@ __global__ void k_rows_round(int *pos, int *wr, int *kvlen, const int *seq_len, 
   if (i == 0) kvlen[b] = ok ? seq_len[b] - 1 + R : 1;  // causal keys 0..n-2+R once the block is written
 }
 
+// rows of a plain decoding step: sequence b's last committed token at position
+// n-1 (blk[b]); keys 0..n-1 once its K/V is written
+__global__ void k_rows_decode(int *pos, int *wr, int *kvlen, int *blk, const int *tokens, const int *seq_len,
+                              const int *active, int batch, int max_ctx, const int *status) {
+  pdl_entry();
+  if (*status) return;
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch) return;
+  const bool ok = active[b] != 0;
+  const int n = seq_len[b];
+  pos[b] = ok ? n - 1 : 0;
+  wr[b] = ok;
+  kvlen[b] = ok ? n : 1;
+  blk[b] = ok ? tokens[(size_t)b * max_ctx + n - 1] : 0;
+}
+
+// after a plain decoding step nothing is carried into a next draft block
+__global__ void k_decode_finish(const int *acc, int *n_carry, int *boundary, int batch, const int *status) {
+  pdl_entry();
+  if (*status) return;
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= batch || acc[b] < 0) return;
+  n_carry[b] = 0;
+  boundary[2 * b] = -1;
+  boundary[2 * b + 1] = -1;
+}
+
 // rows of prefill step c: row b*PF+i at position c0+i if inside the prompt
 __global__ void k_rows_prefill(int *pos, int *wr, int *kvlen, const int *plen, int batch, int c0,
                                const int *status) {
@@ -958,6 +985,35 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   return DFLOW_OK;
 }
 
+// Sec. 5.2 baseline: one greedy step of the target alone (one row per sequence)
+template <typename T>
+dflow_status do_decode(const Call &k, dflow_state *st, int *token_out, int draft_context) {
+  dflow_handle *h = k.h;
+  Dims D = h->D;
+  D.R = 1;
+  const int batch = st->batch;
+  KL(klaunch(k_rows_decode, (batch + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, h->blk, st->tokens,
+             st->seq_len, st->active, batch, h->cfg.max_ctx, k.status));
+  CK(cudaGetLastError());
+  KL(klaunch(k_embed<T>, batch, 256, 0, k.s, (const T *)h->w.embed, h->blk, 1, 1, (const int *)nullptr, h->x, D.d,
+             D.vocab, h->fused ? (T *)h->xn : nullptr, h->tl[0].attn_norm, h->ss, h->rows_max, k.status_w));
+  CK(cudaGetLastError());
+  CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, pick_splits(h, batch, batch)));
+  // commit the prediction: Eq. 3 with no proposals (B = 0) commits exactly the bonus token
+  KL(klaunch(k_accept, (batch + 31) / 32, 32, 0, k.s, h->blk, h->g, (const int *)nullptr, st->tokens, st->seq_len,
+             st->active, batch, 0, h->cfg.max_ctx, h->acc, token_out, k.status_w));
+  CK(cudaGetLastError());
+  if (draft_context) {
+    KL(klaunch(k_carry_rows, (batch + 127) / 128, 128, 0, k.s, h->acc, st->seq_len, batch, 1, h->pos2, h->wr2,
+               k.status));
+    CK(cudaGetLastError());
+    CK(ctx_append<T>(k, D, batch, st, h->feats));
+  }
+  KL(klaunch(k_decode_finish, (batch + 127) / 128, 128, 0, k.s, h->acc, st->n_carry, st->boundary, batch, k.status));
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
 dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
                        int *acc, int *comm) {
   dflow_handle *h = k.h;
@@ -983,14 +1039,16 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
   return DFLOW_OK;
 }
 
-dflow_status guard(const Call &k, dflow_state *st) {
+// device-side checks of the state before a call that writes `rows` rows per sequence
+dflow_status guard_rows(const Call &k, dflow_state *st, int rows) {
   dflow_handle *h = k.h;
   KL(klaunch(k_guard, (st->batch + 127) / 128, 128, 0, k.s, st->tokens, st->seq_len, st->n_carry, st->boundary,
-                                                   st->active, st->batch, h->R, h->cfg.max_ctx,
+                                                   st->active, st->batch, rows, h->cfg.max_ctx,
                                                    h->D.vocab, h->D.B, k.status_w));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
+dflow_status guard(const Call &k, dflow_state *st) { return guard_rows(k, st, k.h->R); }
 
 template <typename T>
 dflow_status do_prefill(const Call &k, dflow_state *st, const int *prompt, int stride, const int *plen_host) {
@@ -1267,6 +1325,17 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
   if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
   if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
   return finish(h, do_carry<float>(k, st, h->blk, h->feats, accept_len, relay));
+}
+
+dflow_status dflow_decode_step(dflow_handle *h, dflow_state *st, int32_t *token_out, int32_t draft_context,
+                               void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!token_out) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  if ((r = guard_rows(k, st, 1))) return finish(h, r);
+  return finish(h, h->dtype == DFLOW_BF16 ? do_decode<bf16>(k, st, token_out, draft_context)
+                                          : do_decode<float>(k, st, token_out, draft_context));
 }
 
 dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable) {

@@ -259,6 +259,13 @@ class Engine:
              ctypes.c_void_p(comm.data_ptr()), int(relay), self._stream())
         return acc, comm
 
+    def decode_step(self, st: DeviceState, draft_context: bool = False, out: Optional[torch.Tensor] = None):
+        """Plain greedy decoding step of the target (the Sec. 5.2 baseline); the committed tokens [batch]."""
+        tok = out if out is not None else self._i32(st.batch)
+        call("dflow_decode_step", self.h, ctypes.byref(st.c), ctypes.c_void_p(tok.data_ptr()), int(draft_context),
+             self._stream())
+        return tok
+
     def profile(self, enable: bool) -> None:
         call("dflow_profile_enable", self.h, int(enable))
 

@@ -239,3 +239,26 @@ def test_batch16_long_context_rounds_stay_clean():
         eng.round(st, torch.as_tensor(sched[r]).cuda())
     assert eng.read_status(st) == 0
     assert np.array_equal(to_np(st.seq_len).astype(np.int64), n0 + (sched + 1).sum(axis=0))
+
+
+def test_full_depth_8b_decode_steps():
+    """The Sec. 5.2 baseline at the benchmark's shape: 2048-token prefill, then
+    64 plain decoding steps (one row through 36 layers, the LM head and its
+    argmax per step).  Every step commits exactly one token, leaves nothing
+    carried and sets no device status; the committed tokens are the target's
+    own predictions (a verify of the same positions reproduces them where the
+    decision is not a near tie)."""
+    from paper_2609_06498_gb300 import Engine, build, random_weights
+    build.build()
+    cfg = synth.QWEN3_8B
+    steps = 64
+    eng = Engine(cfg, random_weights(cfg, seed=0), max_batch=1, max_ctx=cfg.replace(new_tokens=steps + 64).max_ctx())
+    st = eng.new_state(1, page_seed=4)
+    eng.prefill(st, synth.prompts(cfg))
+    assert eng.read_status(st) == 0
+    n0 = int(st.seq_len[0])
+    toks = [int(eng.decode_step(st)[0]) for _ in range(steps)]
+    assert eng.read_status(st) == 0
+    assert int(st.seq_len[0]) == n0 + steps and int(st.n_carry[0]) == 0
+    assert list(to_np(st.tokens)[0, n0:n0 + steps]) == toks
+    assert all(0 <= t < cfg.vocab for t in toks)

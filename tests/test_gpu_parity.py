@@ -273,3 +273,49 @@ def test_long_context_per_call(ctx):
         assert_close(to_np(feats)[b], of, cfg, "features")
         token_check(to_np(g)[b], og, lg)
     assert eng.read_status(st) == 0
+
+
+def test_decode_steps_tiny_equal_plain_greedy():
+    """Sec. 5.2 baseline on the fp32 model: prefill + 24 plain decoding steps
+    through dflow_decode_step give the target's greedy continuation."""
+    from paper_2609_06498_gb300 import Engine, build, pack_weights
+    build.build()
+    cfg = synth.TINY
+    W = synth.weights(cfg)
+    o = Oracle(cfg, W)
+    prompt = synth.prompts(cfg)[0][:40]
+    want = o.greedy_decode(prompt, 25)
+    eng = Engine(cfg, pack_weights(cfg, W), max_batch=1, max_ctx=cfg.max_ctx())
+    st = eng.new_state(1)
+    eng.prefill(st, [prompt])
+    got = [int(st.tokens[0, 40])] + [int(eng.decode_step(st)[0]) for _ in range(24)]
+    assert eng.read_status(st) == 0
+    assert got == list(want)
+    assert int(st.seq_len[0]) == 40 + 25 and int(st.n_carry[0]) == 0
+
+
+def test_decode_step_parity(setup):
+    """dflow_decode_step against Oracle.decode_step from the oracle's state:
+    committed tokens bit exact where the decision is safe, the new K/V rows and
+    (draft_context = 1) the drafter context rows within tolerance."""
+    cfg, W, o, eng = setup
+    ost = _oracle_round_state(cfg, o)
+    st = eng.new_state(cfg.batch, page_seed=9)
+    for step in range(3):
+        upload_state(eng, st, ost)
+        n0 = ost.seq_len.copy()
+        tok = to_np(eng.decode_step(st, draft_context=True))
+        assert eng.read_status(st) == 0
+        for b in range(cfg.batch):
+            want, lg = o.decode_step(ost, b, draft_context=True)
+            token_check([tok[b]], [want], lg[None])
+            n = int(n0[b])
+            assert int(st.seq_len[b]) == n + 1 and int(st.n_carry[b]) == 0
+            k, v = st.read_cache(st.kv, b, n)
+            assert_close(to_np(k)[:, n - 1], ost.k[:, b, n - 1], cfg, "decode K")
+            assert_close(to_np(v)[:, n - 1], ost.v[:, b, n - 1], cfg, "decode V")
+            dk, dv = st.read_cache(st.draft_kv, b, n)
+            assert_close(to_np(dk)[:, n - 1], ost.dk[:, b, n - 1], cfg, "decode ctx K")
+            assert_close(to_np(dv)[:, n - 1], ost.dv[:, b, n - 1], cfg, "decode ctx V")
+            # continue from the oracle's token, whatever a near tie did on the GPU
+            ost.tokens[b, n] = want

@@ -408,6 +408,25 @@ def test_lossless_against_plain_greedy(tiny_oracle):
     assert np.array_equal(toks[0], o.greedy_decode(prompt, TINY.new_tokens))
 
 
+def test_decode_steps_equal_plain_greedy(tiny_oracle):
+    """Sec. 5.2 baseline: cached one-token steps reproduce brute-force greedy
+    decoding (full recompute of every prefix); with draft_context the drafter
+    context equals a fresh recompute of the committed prefix."""
+    o = tiny_oracle
+    prompt = synth.prompts(TINY)[0][:30]
+    st = o.new_state()
+    o.prefill(st, 0, prompt)
+    got = [int(st.tokens[0, 30])] + [o.decode_step(st, 0, draft_context=True)[0] for _ in range(11)]
+    assert got == list(o.greedy_decode(prompt, 12))
+    n = int(st.seq_len[0])
+    assert n == 30 + 12
+    fresh = o.new_state()
+    _, feats = o.target_forward(fresh, 0, st.tokens[0, :n - 1], 0)
+    o.ctx_append(fresh, 0, feats, 0)
+    assert np.allclose(st.dk[:, 0, :n - 1], fresh.dk[:, 0, :n - 1], atol=1e-9)
+    assert np.allclose(st.k[:, 0, :n - 1], fresh.k[:, 0, :n - 1], atol=1e-9)
+
+
 def test_lossless_batch_of_ragged_prompts(tiny_w):
     cfg = TINY.replace(batch=2)
     o = Oracle(cfg, tiny_w)
