@@ -155,7 +155,7 @@ def test_full_width_rounds(name):
             else:
                 gaps = np.concatenate([top2_gap(ro.draft_logits[b][1:]), top2_gap(ro.verify_logits[b])])
                 assert gaps.min() <= 0.05, f"round {r} seq {b}: diverged without a near tie"
-    assert exact >= 2 * cfg.batch and compared >= 1
+    assert exact >= 2 * cfg.batch and (compared >= 1 or cfg.batch == 1)
 
 
 def test_full_depth_8b_round_invariants():
