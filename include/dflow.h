@@ -206,7 +206,9 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
  * carried (n_carry = 0, boundary = -1).  draft_context = 1 also appends the
  * row's Eq. 1 feature to the drafter context, so dflow_round may follow; with
  * 0 (the plain baseline) the drafter context falls behind and no round should
- * follow on that state. */
+ * follow on that state.  The step runs on the block-verify launches with the
+ * anchor in every row of a B+1-row block (rows 1..B are dropped), so it needs
+ * the same free capacity as a round (DFLOW_ERR_CAPACITY otherwise). */
 dflow_status dflow_decode_step(dflow_handle *h, dflow_state *st, int32_t *token_out, int32_t draft_context,
                                void *stream);
 

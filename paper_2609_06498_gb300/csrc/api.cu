@@ -79,28 +79,28 @@ __global__ void k_rows_round(int *pos, int *wr, int *kvlen, const int *seq_len, 
   if (i == 0) kvlen[b] = ok ? seq_len[b] - 1 + R : 1;  // causal keys 0..n-2+R once the block is written
 }
 
-// rows of a plain decoding step: sequence b's last committed token at position
-// n-1 (blk[b]); keys 0..n-1 once its K/V is written
-__global__ void k_rows_decode(int *pos, int *wr, int *kvlen, int *blk, const int *tokens, const int *seq_len,
-                              const int *active, int batch, int max_ctx, const int *status) {
+// block of a plain decoding step: every row of sequence b holds its last
+// committed token (row 0 is the step itself; rows 1..B are computed and dropped)
+__global__ void k_decode_block(int *blk, const int *tokens, const int *seq_len, const int *active, int batch, int R,
+                               int max_ctx, const int *status) {
+  pdl_entry();
+  if (*status) return;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= batch * R) return;
+  const int b = r / R;
+  blk[r] = active[b] ? tokens[(size_t)b * max_ctx + seq_len[b] - 1] : 0;
+}
+
+// after a plain decoding step: the committed token of each sequence (-1 if
+// inactive), and nothing carried into a next draft block
+__global__ void k_decode_finish(const int *acc, const int *comm, int R, int *token_out, int *n_carry, int *boundary,
+                                int batch, const int *status) {
   pdl_entry();
   if (*status) return;
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
-  const bool ok = active[b] != 0;
-  const int n = seq_len[b];
-  pos[b] = ok ? n - 1 : 0;
-  wr[b] = ok;
-  kvlen[b] = ok ? n : 1;
-  blk[b] = ok ? tokens[(size_t)b * max_ctx + n - 1] : 0;
-}
-
-// after a plain decoding step nothing is carried into a next draft block
-__global__ void k_decode_finish(const int *acc, int *n_carry, int *boundary, int batch, const int *status) {
-  pdl_entry();
-  if (*status) return;
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= batch || acc[b] < 0) return;
+  token_out[b] = acc[b] < 0 ? -1 : comm[(size_t)b * R];
+  if (acc[b] < 0) return;
   n_carry[b] = 0;
   boundary[2 * b] = -1;
   boundary[2 * b + 1] = -1;
@@ -461,7 +461,7 @@ struct dflow_handle {
   float *x, *gf32, *apart, *am_val, *ss;
   float2 *rope;
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
-  int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen;
+  int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen, *zeros;
   TcWorkspace tcw;
   DepChain dep;  // completion counters between consecutive tensor-core launches
   // measurement
@@ -540,6 +540,7 @@ size_t layout(dflow_handle *h, char *base) {
   h->comm = (int *)take(rm * 4);
   h->plen = (int *)take((size_t)c.max_batch * 4);
   h->kvlen = (int *)take((size_t)c.max_batch * 4);
+  h->zeros = (int *)take((size_t)c.max_batch * 4);
   h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
   h->dep.dev = (unsigned int *)take(kDepSlots * sizeof(unsigned int));
   const int max_n = std::max(std::max(D.vocab, 2 * D.inter), std::max(h->gld, D.d));
@@ -985,35 +986,6 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   return DFLOW_OK;
 }
 
-// Sec. 5.2 baseline: one greedy step of the target alone (one row per sequence)
-template <typename T>
-dflow_status do_decode(const Call &k, dflow_state *st, int *token_out, int draft_context) {
-  dflow_handle *h = k.h;
-  Dims D = h->D;
-  D.R = 1;
-  const int batch = st->batch;
-  KL(klaunch(k_rows_decode, (batch + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, h->blk, st->tokens,
-             st->seq_len, st->active, batch, h->cfg.max_ctx, k.status));
-  CK(cudaGetLastError());
-  KL(klaunch(k_embed<T>, batch, 256, 0, k.s, (const T *)h->w.embed, h->blk, 1, 1, (const int *)nullptr, h->x, D.d,
-             D.vocab, h->fused ? (T *)h->xn : nullptr, h->tl[0].attn_norm, h->ss, h->rows_max, k.status_w));
-  CK(cudaGetLastError());
-  CK(target_forward<T>(k, D, batch, st, h->g, h->feats, nullptr, pick_splits(h, batch, batch)));
-  // commit the prediction: Eq. 3 with no proposals (B = 0) commits exactly the bonus token
-  KL(klaunch(k_accept, (batch + 31) / 32, 32, 0, k.s, h->blk, h->g, (const int *)nullptr, st->tokens, st->seq_len,
-             st->active, batch, 0, h->cfg.max_ctx, h->acc, token_out, k.status_w));
-  CK(cudaGetLastError());
-  if (draft_context) {
-    KL(klaunch(k_carry_rows, (batch + 127) / 128, 128, 0, k.s, h->acc, st->seq_len, batch, 1, h->pos2, h->wr2,
-               k.status));
-    CK(cudaGetLastError());
-    CK(ctx_append<T>(k, D, batch, st, h->feats));
-  }
-  KL(klaunch(k_decode_finish, (batch + 127) / 128, 128, 0, k.s, h->acc, st->n_carry, st->boundary, batch, k.status));
-  CK(cudaGetLastError());
-  return DFLOW_OK;
-}
-
 dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
                        int *acc, int *comm) {
   dflow_handle *h = k.h;
@@ -1035,6 +1007,30 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
   KL(klaunch(k_carry<T>, dim3(batch, D.B), 256, 0, k.s, (const T *)feats, acc, blk, st->tokens, st->seq_len,
                                                h->cfg.max_ctx, (T *)st->carry, st->n_carry, st->boundary,
                                                D.d, D.B, relay, k.status));
+  CK(cudaGetLastError());
+  return DFLOW_OK;
+}
+
+// Sec. 5.2 baseline: one greedy step of the target alone.  The step runs on the
+// block-verify launches of a round: every row of the block holds the anchor, row
+// 0 is the step (the anchor at position n-1: its K/V, its Eq. 1 feature and its
+// prediction) and rows 1..B are computed and dropped (their K/V lie past the
+// committed length).  At batch 1 every projection streams the same weights for
+// one row or B+1, so the step costs about one verify pass.
+template <typename T>
+dflow_status do_decode(const Call &k, dflow_state *st, int *token_out, int draft_context) {
+  dflow_handle *h = k.h;
+  const int batch = st->batch, R = h->R, rows = batch * R;
+  KL(klaunch(k_decode_block, (rows + 127) / 128, 128, 0, k.s, h->blk, st->tokens, st->seq_len, st->active, batch, R,
+             h->cfg.max_ctx, k.status));
+  CK(cudaGetLastError());
+  dflow_status r;
+  if ((r = do_verify<T>(k, st, h->blk, h->g, h->feats, nullptr))) return r;
+  // commit the prediction of row 0: Eq. 3 with the acceptance forced to 0 commits exactly that token
+  if ((r = do_accept(k, st, h->blk, h->g, h->zeros, h->acc, h->comm))) return r;
+  if (draft_context && (r = do_carry<T>(k, st, h->blk, h->feats, h->acc, 0))) return r;
+  KL(klaunch(k_decode_finish, (batch + 127) / 128, 128, 0, k.s, h->acc, h->comm, R, token_out, st->n_carry,
+             st->boundary, batch, k.status));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
@@ -1239,6 +1235,7 @@ dflow_status dflow_set_workspace(dflow_handle *h, void *dev, size_t bytes) {
   k_rope_table<<<(int)std::min<long long>((n + 255) / 256, 4096), 256>>>(h->rope, h->cfg.max_ctx, h->D.hd,
                                                                           (double)h->cfg.rope_theta);
   CK(cudaGetLastError());
+  CK(cudaMemset(h->zeros, 0, sizeof(int) * h->cfg.max_batch));
   if (h->use_tc) CK(tc_init(h->tcw, 0));
   CK(cudaDeviceSynchronize());
   return DFLOW_OK;
@@ -1333,7 +1330,7 @@ dflow_status dflow_decode_step(dflow_handle *h, dflow_state *st, int32_t *token_
   if (r) return r;
   if (!token_out) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard_rows(k, st, 1))) return finish(h, r);
+  if ((r = guard(k, st))) return finish(h, r);
   return finish(h, h->dtype == DFLOW_BF16 ? do_decode<bf16>(k, st, token_out, draft_context)
                                           : do_decode<float>(k, st, token_out, draft_context));
 }

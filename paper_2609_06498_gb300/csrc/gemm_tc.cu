@@ -1519,7 +1519,7 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
 // The tile schedule of one GEMM of a persistent launch over Q clusters: T
 // tiles, of which the T mod Q left over from the round robin are split over
 // ls = Q / (T mod Q) clusters each, when that divides evenly, every part keeps a
-// k-block and the part slots exist (up to 64 columns: one epilogue chunk per
+// k-block and the part slots exist (32 to 64 columns: one epilogue chunk per
 // owner); cluster q then has nt_a + (q < nt_b) full tiles.
 static void seq_plan(SeqGemm &g, int N, int K, int M, int Q, int npad, bool have_slots) {
   g.N = N;
@@ -1531,7 +1531,7 @@ static void seq_plan(SeqGemm &g, int N, int K, int M, int Q, int npad, bool have
   g.Tf = g.T;
   g.Tl = 0;
   g.ls = 1;
-  if (lo > 0 && npad <= MAX_SPLIT_NPAD && Q <= SEQ_LEFT_MAX && Q % lo == 0 && g.kb >= SEQ_P * (Q / lo) && have_slots) {
+  if (lo > 0 && npad >= 32 && npad <= MAX_SPLIT_NPAD && Q <= SEQ_LEFT_MAX && Q % lo == 0 && g.kb >= SEQ_P * (Q / lo) && have_slots) {
     g.Tf = g.T - lo;
     g.Tl = lo;
     g.ls = Q / lo;

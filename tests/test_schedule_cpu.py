@@ -60,7 +60,7 @@ def check(N, K, M, Q, plan, ctas):
     assert npad % 16 == 0 and M <= npad <= 128 and npad - M < 16 + (16 if npad == 128 else 0)
     assert T == -(-N // BM) and kb == K // BK and Tf + Tl == T and done_n == SEQ_P * T
     if Tl:
-        assert npad <= 64, "leftover split needs one epilogue chunk per owner"
+        assert 32 <= npad <= 64, "leftover split: 32 to 64 columns (one epilogue chunk per owner)"
         assert Tl * ls == Q and Tl == T % Q
     w4 = npad // SEQ_P
     cover = np.zeros((T, kb), np.int32)
@@ -122,11 +122,12 @@ def test_persistent_schedule_covers_every_unit_once(lib, N, K):
 
 def test_schedule_leftover_split_at_the_headline_shapes(lib):
     # Qwen3-8B gate/up (192 tiles) and QKV (48 tiles) on 36 clusters: 12 leftover
-    # tiles each, split over 3 clusters (12 parts of the K range)
+    # tiles each, split over 3 clusters (12 parts of the K range), from 32 columns
     for N in (24576, 6144):
-        for M in (1, 17):
-            code, plan, ctas = schedule(lib, N, 4096, M, 36)
-            assert code == 0 and plan[4] == 12 and plan[5] == 3
+        code, plan, ctas = schedule(lib, N, 4096, 17, 36)
+        assert code == 0 and plan[4] == 12 and plan[5] == 3
+        code, plan, ctas = schedule(lib, N, 4096, 1, 36)
+        assert code == 0 and plan[4] == 0 and plan[3] == plan[1]
     code, _, _ = schedule(lib, 24576, 4096, 68, 36)
     assert code == 0
 
