@@ -574,6 +574,27 @@ def main():
                       "delta_frac": round((on - off) / off, 4),
                       "paper": "0.51 ms, 1.2 % of a DFlash round (Sec. 5.3; A800, model not stated)"}
 
+    # ---- autoregressive baseline (Sec. 5.2, Table 2 "Baseline"): K plain greedy steps of the
+    # target from the same state, one committed token per sequence per step
+    ar = None
+    if rank == 0 and world == 1:
+        wl.restore()
+        tok = torch.empty(cfg.batch, dtype=torch.int32, device="cuda")
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for k in range(K):
+            eng.decode_step(st, draft_context=False, out=tok)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        code = eng.read_status(st)
+        assert code == 0, f"device status {code} set during the autoregressive leg"
+        ar_ms = a0.elapsed_time(a1) / K
+        ar_tps = cfg.batch / (ar_ms / 1e3)
+        ar = {"ms_per_step": round(ar_ms, 4), "tokens_per_s": round(ar_tps, 2),
+              "dflow_speedup": round(value / ar_tps, 3),
+              "note": "one greedy target step per sequence on the block-verify launches (row 0 kept)",
+              "paper": "Table 2, Qwen3-8B conc. 1: DFlow 3.08x AR on GSM8K (A800, trained drafter)"}
+
     # ---- profiled leg: per-launch events around the GEMMs (the dominant kernel)
     wl.restore()
     eng.profile(True)
@@ -610,6 +631,7 @@ def main():
         "phase_ms": {"gemm": round(g["ms"] / K, 4), "attention": round(prof["attn"]["ms"] / K, 4)},
         "step_split_ms": step_split,
         "relay_overhead": relay_cost,
+        "ar_baseline": ar,
         "gpu_launches": int(launches),
         "e2e": e2e,
         "clocks": clocks.summary(),
