@@ -368,18 +368,19 @@ class Oracle:
         st.seq_len[b] = n + a + 1
         return a, committed
 
-    def carry_hidden(self, st: State, b: int, block, feats: np.ndarray, a: int):
+    def carry_hidden(self, st: State, b: int, block, feats: np.ndarray, a: int, relay: bool = True):
         """Sec. 4.2 alignment + Sec. 3 context injection after a commit.
 
         Rows 0..a (anchor and accepted tokens, positions n-1..n-1+a) join the
         drafter context.  Rows a+1..B-1 are carried, shifted by one: next-round
-        slot j takes row a+j.  Boundary tokens are (bonus, y^_{a+1}).
+        slot j takes row a+j.  Boundary tokens are (bonus, y^_{a+1}).  With the
+        relay off (the DFlash baseline of Sec. 5.3) nothing is carried.
         """
         B = self.cfg.block
         n_new = int(st.seq_len[b])
         n_old = n_new - a - 1
         self.ctx_append(st, b, feats[:a + 1], n_old - 1)
-        nc = max(0, B - a - 1)
+        nc = max(0, B - a - 1) if relay else 0
         st.n_carry[b] = nc
         st.carry[b] = 0.0
         for j in range(1, nc + 1):
@@ -412,7 +413,7 @@ class Oracle:
                 blk, out.draft_logits[b], out.draft_x[b] = self.draft_block(st, b)
             g, out.verify_logits[b], feats = self.verify_block(st, b, blk)
             a, comm = self.accept_commit(st, b, blk, g, None if forced is None else forced[b])
-            self.carry_hidden(st, b, blk, feats, a)
+            self.carry_hidden(st, b, blk, feats, a, relay)
             out.block[b], out.g[b], out.feats[b] = blk, g, feats
             out.accept[b], out.committed[b] = a, comm
         return out
