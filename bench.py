@@ -265,6 +265,22 @@ def cpu_baseline_full_round(cfg, timed_sched):
             "sec_per_round": round(sec, 2), "mean_committed_per_round": mean_commit}
 
 
+# DRAM bytes (read + write) per algorithmic byte of the persistent layer-segment
+# GEMM launch, from one ncu capture of it at Qwen3-8B widths and 17 rows
+# (dram__bytes_read.sum + dram__bytes_write.sum = 390.7 MB for 387.3 MB of
+# weights, activations and outputs).  Valid for that kernel as captured.
+SEQ_TRAFFIC_RATIO = {"qwen3_8b_b1": 1.009}
+
+
+def gemm_traffic(cfg, g):
+    """DRAM bytes of the mean GEMM launch of this run, scaled from the capture
+    (traffic grows with the weights streamed), or None without one."""
+    r = SEQ_TRAFFIC_RATIO.get(cfg.name)
+    if r is None or not g["launches"]:
+        return None
+    return round(r * g["bytes"] / g["launches"])
+
+
 def run_cpu_sample(cfg, steps: int, warmup: int, sched):
     s = OracleSample(cfg)
     for w in range(warmup):
