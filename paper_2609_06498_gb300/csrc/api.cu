@@ -711,6 +711,23 @@ EpArgs qkv_ep(const dflow_handle *h, const Dims &D, int nq, const float *qn, con
 
 // attention of one layer: q (h->q) against the layer's pool (and, drafter, the
 // block's own K/V) into h->ao
+AttnArgs layer_attn_args(const dflow_handle *h, void *pool_layer, const dflow_state *st, int causal, int splits) {
+  AttnArgs a{};
+  a.q = h->q;
+  a.pool = pool_layer;
+  a.page_table = st->page_table;
+  a.bk = causal ? nullptr : h->bk;
+  a.bv = causal ? nullptr : h->bv;
+  a.pos = h->pos;
+  a.seq_len = st->seq_len;
+  a.kvlen = h->kvlen;
+  a.causal = causal;
+  a.n_splits = splits;
+  a.part = h->apart;
+  a.out = h->ao;
+  return a;
+}
+
 cudaError_t layer_attention(const Call &k, const Dims &D, int batch, void *pool_layer, const dflow_state *st,
                             int causal, int splits) {
   dflow_handle *h = k.h;
@@ -840,8 +857,11 @@ cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_l
                    h);
   };
   if ((e = gemm(k, Ls[0].w_qkv, qkv_dim, D.d, h->xn, rows, D.d, qkv_args(0)))) return e;
+  // the attention as the first phase of each layer's persistent launch (unless
+  // DFLOW_SEPARATE_ATTENTION asks for its own launch)
+  const bool fuse_attn = seq_attn_supported(D, batch, rows) && getenv("DFLOW_SEPARATE_ATTENTION") == nullptr;
   for (int l = 0; l < nL; ++l) {
-    if ((e = layer_attention(k, D, batch, pool(l), st, causal, splits))) return e;
+    if (!fuse_attn && (e = layer_attention(k, D, batch, pool(l), st, causal, splits))) return e;
     const dflow_layer_weights &L = Ls[l];
     SeqSpec sp[4];
     int n = 0;
@@ -856,7 +876,12 @@ cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_l
     }
     ProfScope ps(h, k.s, DFLOW_PROF_GEMM, bytes, flops);
     ++h->n_launch;
-    if ((e = gemm_seq(h->tcw, n, sp, rows, k.status_w, k.s, &h->dep))) return e;
+    if (fuse_attn) {
+      const SeqAttnSpec as{D, batch, layer_attn_args(h, pool(l), st, causal, splits)};
+      if ((e = gemm_seq(h->tcw, n, sp, rows, k.status_w, k.s, &h->dep, false, &as))) return e;
+    } else if ((e = gemm_seq(h->tcw, n, sp, rows, k.status_w, k.s, &h->dep))) {
+      return e;
+    }
   }
   return cudaSuccess;
 }

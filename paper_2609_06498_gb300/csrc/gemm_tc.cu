@@ -32,6 +32,7 @@
 #include <tuple>
 #include <unordered_map>
 
+#include "attn_t5.cuh"
 #include "gemm_tc.cuh"
 #include "ptx.cuh"
 
@@ -797,6 +798,7 @@ constexpr int SEQ_LEFT_MAX = 40;  // leftover tiles of one GEMM and part slots (
 // and leaves the count at zero again.
 struct SeqGemm {
   int N, K, M, T, kb, mode;
+  int q0, Qg;  // clusters q0 .. q0+Qg-1 take this GEMM's tiles (tile stride Qg)
   int Tf, Tl, ls;
   // the per-CTA schedule without runtime divisions: cluster q has nt_a + (q < nt_b)
   // full tiles; x / ls and x / (SEQ_P ls) are umulhi(x, ls_mag), umulhi(x, parts_mag)
@@ -812,14 +814,27 @@ struct SeqGemm {
 };
 struct SeqMaps {
   CUtensorMap w[SEQ_MAX], x[SEQ_MAX];  // weights [N][K], activations [M][K]
+  CUtensorMap akv, aq;                 // attention phase: one layer of the K/V pool; the query rows (3D)
+};
+// the attention phase ahead of the first GEMM: units u = (kv head u % hkv,
+// sequence u / hkv), unit u on cluster u % n_clusters (its four CTAs are the
+// unit's key splits)
+struct SeqAttnPhase {
+  int on, block, q_tma, n_units, n_clusters;
+  Dims D;
+  AttnArgs a;
+  unsigned int *done;   // each CTA adds 1 per unit it finished
+  unsigned int done_n;  // its value once every unit is finished
 };
 struct SeqParams {
   int n, M, npad, Q, stages, tmem_cols, rx_bytes;
   int independent;  // 1: no GEMM reads another's output; they share the launch's completion counter
   int *status;
-  Dep dep;  // the previous launch: inputs of the first GEMM
+  Dep dep;  // the previous launch: inputs of the first GEMM (and of the attention phase)
+  SeqAttnPhase att;
   SeqGemm g[SEQ_MAX];
 };
+constexpr int SEQ_ATT_KVS = 3;  // K/V pages in flight in the attention phase
 
 // bounded wait on a completion counter (acquire); false on expiry.  The counter
 // holds exactly n once its GEMM is complete (its slot is not reused in the same
@@ -888,19 +903,20 @@ __host__ __device__ __forceinline__ SeqTab seq_tab(const SeqParams &p, int cta) 
   const int q = cta / SEQ_P, rr = cta % SEQ_P;  // cluster, rank in the cluster
 #pragma unroll
   for (int j = 0; j < SEQ_MAX; ++j) {
-    const bool on = j < p.n;
     const SeqGemm &g = p.g[j];
+    const int qj = q - (j < p.n ? g.q0 : 0);  // the cluster's index among the GEMM's clusters
+    const bool on = j < p.n && qj >= 0 && qj < g.Qg;
     const int kb = on ? g.kb : 0;
-    t.t0[j] = q;
-    t.dt[j] = p.Q;
-    t.nt[j] = on ? g.nt_a + (q < g.nt_b ? 1 : 0) : 0;
+    t.t0[j] = on ? qj : 0;
+    t.dt[j] = on ? g.Qg : 1;
+    t.nt[j] = on ? g.nt_a + (qj < g.nt_b ? 1 : 0) : 0;
     t.k0[j] = rr * kb / SEQ_P;
     t.k1[j] = (rr + 1) * kb / SEQ_P;
-    const bool left = on && q < g.Tl * g.ls;
-    const int lt = left ? (int)umulhi32((unsigned)q, g.ls_mag) : 0;
-    const int m = (q - lt * g.ls) * SEQ_P + rr;  // this CTA's part of its leftover tile
+    const bool left = on && qj < g.Tl * g.ls;
+    const int lt = left ? (int)umulhi32((unsigned)qj, g.ls_mag) : 0;
+    const int m = (qj - lt * g.ls) * SEQ_P + rr;  // this CTA's part of its leftover tile
     t.lt[j] = left ? lt : -1;
-    t.lpart[j] = left ? q - lt * g.ls : 0;
+    t.lpart[j] = left ? qj - lt * g.ls : 0;
     t.lk0[j] = left ? (int)umulhi32((unsigned)(m * kb), g.parts_mag) : 0;
     t.lk1[j] = left ? (int)umulhi32((unsigned)((m + 1) * kb), g.parts_mag) : 0;
   }
@@ -946,8 +962,23 @@ __device__ __forceinline__ bool seq_tile(const SeqGemm &g, Smem &sm, float *rx, 
 }
 
 constexpr int SEQ_THREADS = THREADS + 32;  // warp 6: the activation producer
+
+// one unit of the attention phase, out of line so that the phase's registers
+// (a softmax row of 128 O values) do not crowd the GEMM roles'
+__device__ __noinline__ void seq_attn_unit(const SeqMaps &maps, const SeqParams &p, uint8_t *region,
+                                           t5::T5Bars<SEQ_ATT_KVS> &ab, uint32_t tmem, int kvh, int b, int rank,
+                                           const Dep *dep) {
+  if (p.att.block)
+    t5::t5_unit<true, SEQ_P, SEQ_ATT_KVS, SEQ_THREADS>(&maps.akv, &maps.aq, p.att.D, p.att.a, p.att.q_tma, region, ab,
+                                                      tmem, kvh, b, 0, rank, dep, p.status);
+  else
+    t5::t5_unit<false, SEQ_P, SEQ_ATT_KVS, SEQ_THREADS>(&maps.akv, &maps.aq, p.att.D, p.att.a, p.att.q_tma, region, ab,
+                                                       tmem, kvh, b, 0, rank, dep, p.status);
+}
 // the CTA's schedule in shared memory, after the Smem block
 constexpr size_t SEQ_SMEM_TAB_OFF = (sizeof(Smem) + 15) & ~(size_t)15;
+// after the schedule: the attention phase's barriers and per-row results
+constexpr size_t SEQ_SMEM_ATT_OFF = (SEQ_SMEM_TAB_OFF + sizeof(SeqTab) + 15) & ~(size_t)15;
 
 // NPAD: the token columns (p.npad, seq_npad), a compile-time constant so that
 // the split-K epilogue has fixed trip counts
@@ -1001,6 +1032,28 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
 
+  // ---------------- attention phase (clusters 0 .. n_clusters - 1) ----------------
+  // The ring and the receive area hold the units' Q, K/V pages and P tiles; this
+  // CTA's weight stream starts after it.  The first GEMM's activations are the
+  // phase's output: its activation producer waits for the phase's count.
+  if (p.att.on) {
+    const int q = (int)blockIdx.x / SEQ_P;
+    if (q < p.att.n_clusters) {
+      t5::T5Bars<SEQ_ATT_KVS> &ab =
+          *reinterpret_cast<t5::T5Bars<SEQ_ATT_KVS> *>(reinterpret_cast<uint8_t *>(&sm) + SEQ_SMEM_ATT_OFF);
+      const Dep *dep = &p.dep;
+      for (int u = q; u < p.att.n_units; u += p.att.n_clusters) {
+        const int kvh = u % p.att.D.hkv, b = u / p.att.D.hkv;
+        seq_attn_unit(maps, p, ring, ab, tmem, kvh, b, rank, dep);
+        dep = nullptr;
+        if (threadIdx.x == 0) counter_add(p.att.done, 1u);  // after the unit's closing cluster barrier
+      }
+      tc_fence_before();
+      __syncthreads();
+      tc_fence_after();
+    }
+  }
+
   if (warp == 0 || warp == 6) {
     // ---------------- TMA producers: warp 0 streams every unit's weight k-block
     // (nothing to wait for but a free stage, so the next GEMM's weights fill the
@@ -1022,7 +1075,14 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
         const CUtensorMap *map = wp ? seq_wmap(maps, j) : seq_xmap(maps, j);
         if (!wp) {
           // GEMM j reads what GEMM j - 1 (or the previous launch) wrote
-          if (j == 0 || p.independent) {
+          if (j == 0 && p.att.on) {
+            // the attention phase's output (it waited for the launch's inputs itself)
+            if (!counter_wait(p.att.done, p.att.done_n, p.status)) {
+              ok = false;
+              break;
+            }
+            dep_done = true;
+          } else if (j == 0 || p.independent) {
             // the launch's inputs: once, before this producer's first copy
             if (!dep_done) dep_wait(p.dep, p.status);
             dep_done = true;
@@ -1030,7 +1090,7 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
             ok = false;
             break;
           }
-          if ((j > 0 && !p.independent) || p.dep.wait) fence_proxy_async_global();
+          if ((j > 0 && !p.independent) || p.dep.wait || (j == 0 && p.att.on)) fence_proxy_async_global();
           prefetch_tensormap(map);
         }
         // the leftover part first, then the full tiles
@@ -1316,7 +1376,7 @@ size_t seq_smem(int npad, int *stages_out, int *rx_bytes_out) {
   const int stage_bytes = A_BYTES + npad * BK * 2;
   // receive area of the 4-way split: a [BM][npad / 4] fp32 slot per rank
   const size_t red_bytes = (size_t)SEQ_P * BM * (npad / SEQ_P) * 4;
-  const size_t tail = SEQ_SMEM_TAB_OFF + sizeof(SeqTab);  // Smem, then the schedule
+  const size_t tail = SEQ_SMEM_ATT_OFF + sizeof(t5::T5Bars<SEQ_ATT_KVS>);  // Smem, schedule, attention barriers
   int stages = (int)((SMEM_BUDGET - red_bytes - tail - 1024) / stage_bytes);
   if (stages > 16) stages = 16;
   *stages_out = stages;
@@ -1521,7 +1581,9 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
 // ls = Q / (T mod Q) clusters each, when that divides evenly, every part keeps a
 // k-block and the part slots exist (32 to 64 columns: one epilogue chunk per
 // owner); cluster q then has nt_a + (q < nt_b) full tiles.
-static void seq_plan(SeqGemm &g, int N, int K, int M, int Q, int npad, bool have_slots) {
+static void seq_plan(SeqGemm &g, int N, int K, int M, int Q, int npad, bool have_slots, int q0 = 0) {
+  g.q0 = q0;
+  g.Qg = Q;
   g.N = N;
   g.K = K;
   g.M = M;
@@ -1560,9 +1622,15 @@ static bool same_qkv_table(const QkvOut &a, const QkvOut &b) {
          (a.bk == nullptr) == (b.bk == nullptr);
 }
 
+bool seq_attn_supported(const Dims &D, int batch, int M) {
+  return D.hd == 128 && D.page_size == 64 && D.R * (D.hq / D.hkv) <= t5::T5_ROWS && batch >= 1 &&
+         seq_supported(M);
+}
+
 cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
-                     DepChain *chain, bool independent) {
+                     DepChain *chain, bool independent, const SeqAttnSpec *att) {
   if (n < 1 || n > SEQ_MAX || !chain || !chain->dev || !seq_supported(M)) return cudaErrorInvalidValue;
+  if (att && (independent || !seq_attn_supported(att->D, att->batch, M))) return cudaErrorInvalidValue;
   SeqParams p{};
   SeqMaps maps{};
   p.n = n;
@@ -1576,6 +1644,31 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
   const size_t smem = seq_smem(p.npad, &p.stages, &p.rx_bytes);
   p.Q = seq_clusters(p.npad, smem);
   if (p.Q < 1 || p.stages < 3) return cudaErrorInvalidValue;
+  int q0_first = 0, qn_first = p.Q;  // clusters of the first GEMM
+  if (att) {
+    // the attention phase: its region is the ring and the receive area
+    if ((size_t)p.stages * (A_BYTES + p.npad * BK * 2) + p.rx_bytes < t5::t5_region_bytes<SEQ_ATT_KVS>())
+      return cudaErrorInvalidValue;
+    const Dims &D = att->D;
+    const int G = D.hq / D.hkv;
+    SeqAttnPhase &at = p.att;
+    at.on = 1;
+    at.block = att->a.causal ? 0 : 1;
+    at.D = D;
+    at.a = att->a;
+    at.n_units = D.hkv * att->batch;
+    at.n_clusters = at.n_units < p.Q ? at.n_units : p.Q;
+    if (!tensor_map(&maps.akv, att->a.pool, D.num_pages * 2 * D.hkv * D.page_size, D.hd, D.hd, 64))
+      return cudaErrorInvalidValue;
+    at.q_tma = tensor_map_3d(&maps.aq, att->a.q, D.hd, D.hq, att->batch * D.R, G, D.R) ? 1 : 0;
+    if (p.tmem_cols < t5::T5_TMEM_COLS) p.tmem_cols = t5::T5_TMEM_COLS;
+    // the phase on the first clusters (placed first); the first GEMM (it reads the
+    // phase's output) on the others when they are the majority
+    if (2 * at.n_clusters <= p.Q) {
+      q0_first = at.n_clusters;
+      qn_first = p.Q - at.n_clusters;
+    }
+  }
   const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(p.npad >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
   for (int j = 0; j < n; ++j) {
     const SeqSpec &q = sp[j];
@@ -1588,7 +1681,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
       return cudaErrorInvalidValue;
     SeqGemm &g = p.g[j];
     g.mode = mode;
-    seq_plan(g, q.N, q.K, M, p.Q, p.npad, w.lacc != nullptr);
+    seq_plan(g, q.N, q.K, M, j == 0 ? qn_first : p.Q, p.npad, w.lacc != nullptr, j == 0 ? q0_first : 0);
     if (g.Tl > 0) {
       g.lacc = w.lacc + (size_t)j * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD;
       g.lctr = w.lctr + (size_t)j * SEQ_LEFT_MAX * SEQ_P;
@@ -1600,6 +1693,7 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
       return cudaErrorInvalidValue;
   }
   auto done_count = [&](const SeqGemm &g) { return (unsigned)(SEQ_P * g.T); };  // each owner once per tile
+  if (att) p.att.done = chain->alloc((unsigned)(SEQ_P * p.att.n_units), &p.att.done_n);  // each CTA once per unit
   if (independent) {
     // no GEMM waits for another: every GEMM counts into the launch's counter
     unsigned total = 0;

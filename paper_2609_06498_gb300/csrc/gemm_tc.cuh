@@ -47,13 +47,24 @@ struct SeqSpec {
 };
 // True when up to 4 GEMMs over M rows can run as one persistent launch.
 bool seq_supported(int M);
+// The attention of one layer, run as the first phase of a persistent launch
+// whose first GEMM reads its output (the O projection).
+struct SeqAttnSpec {
+  Dims D;     // D.R: rows per sequence
+  int batch;
+  AttnArgs a;  // q, pool (this layer), page table, block K/V (drafter), pos, seq_len, kvlen, causal, out
+};
+// True when the attention can be such a phase: 128-dim heads, 64-token pages,
+// one 128-row group of query rows per (kv head, sequence), M <= 128 rows.
+bool seq_attn_supported(const Dims &D, int batch, int M);
 // The GEMMs of `sp` in order, in one launch: GEMM j's activations are read once
 // every tile of GEMM j - 1 is finished; the first waits for the previous launch
 // in `chain` (required), the next launch waits for the last GEMM.  independent:
 // no GEMM reads another's output (all wait only for the previous launch; the next
 // launch waits for all of them); Q/K/V epilogues may then appear more than once
 // if they share their column table.
+// att: the attention phase ahead of the first GEMM (not with independent), or null.
 cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int *status, cudaStream_t s,
-                     DepChain *chain, bool independent = false);
+                     DepChain *chain, bool independent = false, const SeqAttnSpec *att = nullptr);
 
 }  // namespace dflow

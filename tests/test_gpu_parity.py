@@ -213,6 +213,16 @@ def test_round_parity_separate_gemms(setup, monkeypatch):
     test_round_parity(setup, True)
 
 
+def test_round_parity_separate_attention(setup, monkeypatch):
+    """The same rounds with the attention in its own launch instead of as the
+    first phase of each layer's persistent launch."""
+    cfg = setup[0]
+    if cfg.dtype != "bf16" or cfg.head_dim != 128:
+        pytest.skip("the fused attention phase is the bf16 path with 128-dim heads")
+    monkeypatch.setenv("DFLOW_SEPARATE_ATTENTION", "1")
+    test_round_parity(setup, True)
+
+
 def test_generate_matches_oracle_tiny():
     """fp32: the whole generation (prefill + natural-acceptance rounds) equals the
     oracle's, which the oracle tests pin to plain greedy decoding."""
