@@ -1051,6 +1051,8 @@ k_gemm_seq(const __grid_constant__ SeqMaps maps, const __grid_constant__ SeqPara
       tc_fence_before();
       __syncthreads();
       tc_fence_after();
+      // the weight copies that now refill the ring follow the phase's own accesses to it
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
   }
 
