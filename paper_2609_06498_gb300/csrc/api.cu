@@ -857,9 +857,12 @@ cudaError_t stack_forward(const Call &k, const Dims &D, int batch, const dflow_l
                    h);
   };
   if ((e = gemm(k, Ls[0].w_qkv, qkv_dim, D.d, h->xn, rows, D.d, qkv_args(0)))) return e;
-  // the attention as the first phase of each layer's persistent launch (unless
-  // DFLOW_SEPARATE_ATTENTION asks for its own launch)
-  const bool fuse_attn = seq_attn_supported(D, batch, rows) && getenv("DFLOW_SEPARATE_ATTENTION") == nullptr;
+  // DFLOW_FUSED_ATTENTION: the attention as the first phase of each layer's
+  // persistent launch instead of its own launch (same results; at batch 1 the
+  // separate launch is faster: its start overlaps the previous launch's tail and
+  // it uses twice the key splits, while in the fused launch the attention
+  // clusters join the gate/up projection late)
+  const bool fuse_attn = seq_attn_supported(D, batch, rows) && getenv("DFLOW_FUSED_ATTENTION") != nullptr;
   for (int l = 0; l < nL; ++l) {
     if (!fuse_attn && (e = layer_attention(k, D, batch, pool(l), st, causal, splits))) return e;
     const dflow_layer_weights &L = Ls[l];

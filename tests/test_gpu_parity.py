@@ -213,13 +213,13 @@ def test_round_parity_separate_gemms(setup, monkeypatch):
     test_round_parity(setup, True)
 
 
-def test_round_parity_separate_attention(setup, monkeypatch):
-    """The same rounds with the attention in its own launch instead of as the
-    first phase of each layer's persistent launch."""
+def test_round_parity_fused_attention(setup, monkeypatch):
+    """The same rounds with the attention as the first phase of each layer's
+    persistent launch instead of its own launch."""
     cfg = setup[0]
     if cfg.dtype != "bf16" or cfg.head_dim != 128:
         pytest.skip("the fused attention phase is the bf16 path with 128-dim heads")
-    monkeypatch.setenv("DFLOW_SEPARATE_ATTENTION", "1")
+    monkeypatch.setenv("DFLOW_FUSED_ATTENTION", "1")
     test_round_parity(setup, True)
 
 
