@@ -236,7 +236,8 @@ dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable);
  * library's GEMM kernels (path 0: CUDA-core kernel of fp32 handles; bf16
  * handles: path 1 the tcgen05 kernel of one projection, path 2 the persistent
  * tcgen05 launch the round uses for up to 128 rows (modes 0-3, K a multiple of
- * 64 and at least 256); else DFLOW_ERR_UNSUPPORTED), with the epilogue `mode`: 0 store fp32 out[M][ldo];
+ * 64 and at least 256), path 3 the one-pass tcgen05 launch the round uses above
+ * 128 rows; else DFLOW_ERR_UNSUPPORTED), with the epilogue `mode`: 0 store fp32 out[M][ldo];
  * 1 add into fp32 out[M][ldo]; 2 SwiGLU of 128-row [64 gate | 64 up] groups
  * into model-dtype out[M][ldo] (N/2 features); 3 SiLU into model-dtype out;
  * 4 greedy argmax over n into int32 out[M] (M <= max_batch * max(B+1, 64)).

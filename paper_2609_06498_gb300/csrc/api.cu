@@ -612,6 +612,8 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
     return gemm_seq(h->tcw, 1, &sp, M, k.status_w, k.s, &h->dep);
   }
   if (!tc_supports(N, K, M, ldx, ep)) return cudaErrorInvalidValue;
+  // more rows than the persistent launch takes: one pass over the weights for up to 512 rows
+  if (M > 128) return gemm_wide(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, &h->dep);
   return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
 }
 
@@ -1391,7 +1393,7 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
                               int32_t M, int32_t ldx, int32_t mode, void *out, int32_t ldo, int32_t *status,
                               void *stream) {
   if (!h || !h->ws || !W || !X || !out || !status || N < 1 || K < 1 || M < 1 || ldx < K) return DFLOW_ERR_INVALID_ARG;
-  if ((path >= 1) != (h->dtype == DFLOW_BF16) || path < 0 || path > 2) return DFLOW_ERR_UNSUPPORTED;
+  if ((path >= 1) != (h->dtype == DFLOW_BF16) || path < 0 || path > 3) return DFLOW_ERR_UNSUPPORTED;
   if (path == 2 && (mode == EP_ARGMAX || K % 64 || K / 64 < 4 || ldx % 8 || !seq_supported(M)))
     return DFLOW_ERR_UNSUPPORTED;
   if (mode < 0 || mode > 4) return DFLOW_ERR_INVALID_ARG;
@@ -1420,6 +1422,8 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
     e = gemm_seq(h->tcw, 1, &sp, M, status, s, &h->dep);
     h->dep.brk();
     if (e != cudaSuccess) h->dep.dirty = true;
+  } else if (path == 3) {
+    e = gemm_wide(h->tcw, W, N, K, X, M, ldx, ep, status, s);
   } else if (path == 1) {
     e = tc_supports(N, K, M, ldx, ep) ? gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, status, s) : cudaErrorNotSupported;
   } else {

@@ -45,7 +45,8 @@ using namespace ptx;
 constexpr int BM = 128;           // weight rows per tile (MMA M)
 constexpr int BK = 64;            // k elements per k-block (128 bytes of bf16: one swizzle row)
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int MAX_NPAD = 256;
+constexpr int MAX_NPAD = 256;    // token columns of one k_gemm_tc pass (one MMA's N)
+constexpr int MAX_COLS = 512;    // token columns of the per-column tables (k_gemm_wide: two MMAs per k-step)
 constexpr int MAX_SPLIT_NPAD = 64;  // split-K (P > 1) only for up to 64 token columns
 constexpr int SEQ_MAX_NPAD = 128;   // token columns of the persistent layer-segment kernel
 constexpr int THREADS = 192;
@@ -72,9 +73,9 @@ struct Smem {
   float rv[4][16];
   int ri[4][16];
   float ssred[4][16];
-  float col_scale[MAX_NPAD];
-  long long qkv_base[MAX_NPAD];  // EP_QKV, paged pool: element offset of the column's K slot of kv head 0, or -1
-  int qkv_pos[MAX_NPAD];         // EP_QKV: position of the column's row
+  float col_scale[MAX_COLS];
+  long long qkv_base[MAX_COLS];  // EP_QKV, paged pool: element offset of the column's K slot of kv head 0, or -1
+  int qkv_pos[MAX_COLS];         // EP_QKV: position of the column's row
 };
 
 // epilogue inputs that do not depend on the product, loaded while the MMAs run
@@ -217,7 +218,7 @@ __device__ __forceinline__ void epilogue_chunk(const PT &p, Smem &sm, int t, int
   const int cend = min(c0 + nc, p.M);
   if (ep.in_ss) {
 #pragma unroll
-    for (int j = 0; j < NC; ++j) v[j] *= sm.col_scale[min(c0 + j, MAX_NPAD - 1)];
+    for (int j = 0; j < NC; ++j) v[j] *= sm.col_scale[min(c0 + j, MAX_COLS - 1)];
   }
   if constexpr (EP == EP_STORE_F32 || EP == EP_SILU) {
     if (n < p.N) {
@@ -765,6 +766,254 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
   __syncthreads();
   if (threadIdx.x == 0) dep_signal(p.dep);  // every global write of this CTA is done
   if (p.P > 1) cluster_sync();  // no CTA leaves while a peer may still read its shared memory
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
+  }
+}
+
+// ===========================================================================
+// Wide weight-streaming GEMM: up to 512 token rows in one pass over the weights
+// (two MMAs per k-step once the padded rows exceed one MMA's N of 256), for the
+// blocks of large batches.  The grid is Q tile groups x P k-splits of
+// independent CTAs: CTA (q, r) takes tiles q, q + Q, ... over k-blocks
+// [r kb / P, (r + 1) kb / P).  With P > 1 each CTA stores its fp32 partial of
+// a tile in an L2 slot; the CTA whose arrival completes the tile's count adds
+// the P slots in rank order (so the result does not depend on the arrival
+// order), runs the fused epilogue and leaves the count at zero.
+// ===========================================================================
+constexpr int WIDE_MAX_NPAD = 512;
+constexpr int WIDE_MAX_TILES = 4096;                    // 128-row tiles of one projection (N <= 524288)
+constexpr size_t WIDE_SLOT_BYTES = (size_t)48 << 20;   // split-K partials, kept well inside L2
+
+struct WideParams {
+  int N, K, M, npad, T, kb, P, Q, stages, tmem_cols, nbuf;
+  uint32_t idesc1, idesc2;  // MMA N = min(npad, 256), and npad - 256
+  EpArgs ep;
+  int *status;
+  Dep dep;
+  float *slots;       // [T][P][BM][npad] partials (P > 1)
+  unsigned int *ctr;  // [T] arrivals per tile (zero between uses)
+};
+
+template <int EP>
+__global__ void __launch_bounds__(THREADS, 1)
+k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX1,
+            const __grid_constant__ CUtensorMap tmX2, const WideParams p) {
+  // the next kernel may launch once every CTA of this one runs; inputs produced by
+  // the previous launch are read only after dep_wait() (weights are prefetched before it)
+  pdl_trigger();
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  uint8_t *ring = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
+  const int stage_bytes = A_BYTES + p.npad * BK * 2;
+  Smem &sm = *reinterpret_cast<Smem *>(ring + (size_t)p.stages * stage_bytes);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int q = (int)blockIdx.x / p.P, rank = (int)blockIdx.x % p.P;
+  const int kr0 = rank * p.kb / p.P, kr1 = (rank + 1) * p.kb / p.P;
+  const bool two = p.npad > 256;  // a second MMA (and X box) for rows 256..npad-1
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&sm.accf[b], 1);
+      mbar_init(&sm.acce[b], 4);
+    }
+    mbar_init(&sm.drain, 1);
+    sm.abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
+                 "r"(p.tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem;
+  const int n_tiles = q < p.T ? (p.T - q + p.Q - 1) / p.Q : 0;  // tiles of this CTA
+
+  if (warp == 0) {
+    // ---------------- TMA producer ----------------
+    if (lane == 0) {
+      const uint64_t pw = policy_evict_first(), px = policy_evict_last();
+      const int nk = kr1 - kr0, n_units = n_tiles * nk;
+      auto load_x = [&](uint8_t *a, int k, uint64_t *bar) {
+        tma_load_2d(a + A_BYTES, &tmX1, k * BK, 0, bar, px);
+        if (two) tma_load_2d(a + A_BYTES + 256 * 128, &tmX2, k * BK, 256, bar, px);
+      };
+      int n_issued = 0;
+      bool ok = true;
+      // weight tiles of the first ring do not depend on the previous kernel: start them now
+      const int pre = n_units < p.stages ? n_units : p.stages;
+      for (int u = 0; u < pre; ++u) {
+        mbar_expect_tx(&sm.full[u], stage_bytes);
+        tma_load_2d(ring + (size_t)u * stage_bytes, &tmW, (kr0 + u % nk) * BK, (q + (u / nk) * p.Q) * BM, &sm.full[u], pw);
+      }
+      n_issued = pre;
+      dep_wait(p.dep, p.status);
+      if (p.dep.wait) fence_proxy_async_global();
+      for (int u = 0; u < pre; ++u) load_x(ring + (size_t)u * stage_bytes, kr0 + u % nk, &sm.full[u]);
+      int stage = pre % p.stages;
+      uint32_t ph = pre == p.stages ? 1 : 0;
+      for (int u = pre; u < n_units; ++u) {
+        const int t = q + (u / nk) * p.Q, k = kr0 + u % nk;
+        if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
+          ok = false;
+          break;
+        }
+        uint8_t *a = ring + (size_t)stage * stage_bytes;
+        mbar_expect_tx(&sm.full[stage], stage_bytes);
+        tma_load_2d(a, &tmW, k * BK, t * BM, &sm.full[stage], pw);
+        load_x(a, k, &sm.full[stage]);
+        n_issued = u + 1;
+        if (++stage == p.stages) {
+          stage = 0;
+          ph ^= 1;
+        }
+      }
+      if (!ok) {
+        set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+        atomicExch(&sm.abort, 1);
+      }
+      // every copy this thread started has landed before the CTA may exit
+      for (int u = n_issued > p.stages ? n_issued - p.stages : 0; u < n_issued; ++u)
+        if (!mbar_wait(&sm.full[u % p.stages], (uint32_t)((u / p.stages) & 1)))
+          set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (int i = 0; i < n_tiles && ok; ++i) {
+        const int buf = p.nbuf == 2 ? (i & 1) : 0;
+        const uint32_t par = p.nbuf == 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
+        if (!mbar_wait(&sm.acce[buf], par ^ 1)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d = tmem + buf * p.npad;
+        for (int k = kr0; k < kr1; ++k) {
+          if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a = smem_u32(ring + (size_t)stage * stage_bytes);
+          const uint64_t ad = smem_desc(a), bd1 = smem_desc(a + A_BYTES), bd2 = smem_desc(a + A_BYTES + 256 * 128);
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint32_t acc = (k > kr0 || kk > 0) ? 1u : 0u;
+            mma_bf16(d, ad + 2 * kk, bd1 + 2 * kk, p.idesc1, acc);
+            if (two) mma_bf16(d + 256, ad + 2 * kk, bd2 + 2 * kk, p.idesc2, acc);
+          }
+          mma_commit(&sm.empty[stage]);
+          if (++stage == p.stages) {
+            stage = 0;
+            ph ^= 1;
+          }
+        }
+        if (!ok) break;
+        mma_commit(&sm.accf[buf]);
+      }
+      if (!ok) {
+        set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+        atomicExch(&sm.abort, 1);
+      }
+      mma_commit(&sm.drain);
+      if (!mbar_wait(&sm.drain, 0)) set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+    }
+  } else {
+    // ---------------- epilogue warps 2..5 ----------------
+    const int sub = warp & 3;
+    const int r = sub * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(sub * 32) << 16);
+    const bool leader = threadIdx.x == 64;
+    if (leader) dep_wait(p.dep, p.status);
+    epi_bar();
+    if (p.ep.in_ss) col_scales(p.ep, sm, p.M, r);
+    if constexpr (EP == EP_QKV) {
+      qkv_table(p.ep.qkv, sm, p.M, r);
+      epi_bar();
+    }
+    const int cols = p.npad < p.M ? p.npad : p.M;
+    for (int i = 0; i < n_tiles; ++i) {
+      const int t = q + i * p.Q;
+      const int buf = p.nbuf == 2 ? (i & 1) : 0;
+      const uint32_t par = p.nbuf == 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
+      EpPre pre;
+      if (p.P == 1) epilogue_prefetch<EP>(p, sm, t, r, 0, 16, pre);
+      if (leader) sm.flag = mbar_wait(&sm.accf[buf], par) ? 1 : 0;
+      __syncwarp();
+      epi_bar();
+      if (!sm.flag) {
+        if (leader) {
+          set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+          atomicExch(&sm.abort, 1);
+        }
+        break;
+      }
+      tc_fence_after();
+      const uint32_t acc_addr = lane_addr + buf * p.npad;
+      float v[16];
+      if (p.P == 1) {
+        for (int c0 = 0; c0 < cols; c0 += 16) {
+          if (c0 > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
+          tmem_ld16(acc_addr + c0, v);
+          epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v, pre);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.acce[buf]);
+      } else {
+        // this CTA's partial of row r into its slot, then free the accumulator
+        float *const mine = p.slots + (((size_t)t * p.P + rank) * BM + r) * p.npad;
+        for (int c0 = 0; c0 < cols; c0 += 16) {
+          tmem_ld16(acc_addr + c0, v);
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4)
+            __stcg(reinterpret_cast<float4 *>(mine + c0 + 4 * q4),
+                   make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.acce[buf]);
+        // the leader's count is a release at GPU scope after every thread's stores
+        // (through the barrier), and an acquire for the last arriver's reads
+        epi_bar();
+        if (leader) sm.left_last = atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(p.P - 1) ? 1 : 0;
+        epi_bar();
+        if (sm.left_last) {
+          const float *const row0 = p.slots + ((size_t)t * p.P * BM + r) * p.npad;
+          const size_t rstride = (size_t)BM * p.npad;
+          for (int c0 = 0; c0 < cols; c0 += 16) {
+            epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = 0.f;
+            for (int rr = 0; rr < p.P; ++rr) {
+#pragma unroll
+              for (int q4 = 0; q4 < 4; ++q4) {
+                const float4 y = __ldcg(reinterpret_cast<const float4 *>(row0 + rr * rstride + c0 + 4 * q4));
+                v[4 * q4] += y.x;
+                v[4 * q4 + 1] += y.y;
+                v[4 * q4 + 2] += y.z;
+                v[4 * q4 + 3] += y.w;
+              }
+            }
+            epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v, pre);
+          }
+          if (leader) *reinterpret_cast<volatile unsigned int *>(p.ctr + t) = 0u;
+        }
+      }
+      epi_bar();  // sm.flag and sm.left_last are rewritten at the next tile
+    }
+  }
+
+  __syncwarp();  // lanes that skipped a single-thread role wait for it here
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0) dep_signal(p.dep);  // every global write of this CTA is done
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(p.tmem_cols) : "memory");
@@ -1506,17 +1755,24 @@ bool tensor_map_3d(CUtensorMap *out, const void *ptr, int d0, int d1, int d2, in
 }
 
 void tc_layout(TcWorkspace &w, char *base, size_t &off, int sm_count, size_t rows_max, int max_tiles) {
-  (void)rows_max;
-  (void)max_tiles;
   w.sm_count = sm_count;  // split-K partials of whole tiles stay in distributed shared memory
   // the persistent launch's leftover-tile sums and counts, per GEMM slot
   off = (off + 255) & ~(size_t)255;
   const size_t acc_bytes = (size_t)SEQ_MAX * SEQ_LEFT_MAX * BM * MAX_SPLIT_NPAD * sizeof(float);
   const size_t ctr_bytes = (size_t)SEQ_MAX * SEQ_LEFT_MAX * SEQ_P * sizeof(unsigned int);
+  const size_t wctr_bytes = (size_t)WIDE_MAX_TILES * sizeof(unsigned int);
   w.lacc = base ? reinterpret_cast<float *>(base + off) : nullptr;
   w.lctr = base ? reinterpret_cast<unsigned int *>(base + off + acc_bytes) : nullptr;
-  w.left_bytes = acc_bytes + ctr_bytes;
+  w.wctr = base ? reinterpret_cast<unsigned int *>(base + off + acc_bytes + ctr_bytes) : nullptr;
+  w.left_bytes = acc_bytes + ctr_bytes + wctr_bytes;
   off += (w.left_bytes + 255) & ~(size_t)255;
+  // the wide launch's split-K partials: at most WIDE_SLOT_BYTES, and never more
+  // than every tile of the widest projection for rows_max rows in 4 parts
+  const int max_cols = (int)(rows_max < (size_t)WIDE_MAX_NPAD ? (rows_max + 15) / 16 * 16 : WIDE_MAX_NPAD);
+  size_t want = (size_t)max_tiles * 4 * BM * max_cols * sizeof(float);
+  w.wslot_bytes = want < WIDE_SLOT_BYTES ? want : WIDE_SLOT_BYTES;
+  w.wslots = base ? reinterpret_cast<float *>(base + off) : nullptr;
+  off += (w.wslot_bytes + 255) & ~(size_t)255;
 }
 
 bool tc_supports(int N, int K, int M, int ldx, const EpArgs &ep) {
@@ -1571,6 +1827,137 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
       case EP_SILU: e = run<EP_SILU>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
       case EP_ARGMAX: e = run<EP_ARGMAX>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
       case EP_QKV: e = run<EP_QKV>(mw, mx, p, w.sm_count, s, use_caches, chain); break;
+      default: e = cudaErrorInvalidValue;
+    }
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+namespace {
+
+inline uint32_t mma_idesc(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+}
+
+struct WideChoice {
+  int P = 0, Q = 0, stages = 0;
+  size_t smem = 0;
+};
+
+// k-splits and tile groups minimising the k-blocks each CTA streams, with a
+// charge for writing a split tile's partial to L2 and for the last arriver
+// reading the P partials back (both in k-block equivalents at L2 speed)
+WideChoice choose_wide(int T, int kb, int npad, int sms, size_t slot_bytes) {
+  WideChoice best;
+  const int stage_bytes = A_BYTES + npad * BK * 2;
+  int stages = (int)((SMEM_BUDGET - sizeof(Smem) - 1024) / stage_bytes);
+  if (stages > 16) stages = 16;
+  if (stages < 2) return best;
+  const int part_kb = (npad * BM * 4 / (3 * A_BYTES)) + 1;  // one partial tile, in k-blocks at about 3x
+  long best_cost = -1;
+  for (int P : {1, 2, 3, 4, 6, 8}) {
+    if (P > 1 && (kb / P < 2 || (size_t)T * P * BM * npad * sizeof(float) > slot_bytes)) continue;
+    int Q = sms / P;
+    if (Q < 1) continue;
+    if (Q > T) Q = T;
+    const long rounds = (T + Q - 1) / Q;
+    const long cost = rounds * ((kb + P - 1) / P) + (P > 1 ? (long)part_kb * (1 + P) : 0);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best.P = P;
+      best.Q = Q;
+    }
+  }
+  best.stages = stages;
+  best.smem = 1024 + (size_t)stages * stage_bytes + sizeof(Smem);
+  return best;
+}
+
+template <int EP>
+cudaError_t launch_wide(const CUtensorMap &mw, const CUtensorMap &mx1, const CUtensorMap &mx2, const WideParams &p,
+                        size_t smem, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_wide<EP>, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BUDGET + 2048);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.P * p.Q);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_gemm_wide<EP>, mw, mx1, mx2, p);
+}
+
+}  // namespace
+
+cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
+                      const EpArgs &ep_in, int *status, cudaStream_t s, DepChain *chain) {
+  if (N < 1 || K < BK || K % BK || M < 1 || ldx % 8 || (N + BM - 1) / BM > WIDE_MAX_TILES || w.wctr == nullptr)
+    return cudaErrorInvalidValue;
+  CUtensorMap mw;
+  if (!tensor_map(&mw, W, N, K, K, BM)) return cudaErrorInvalidValue;
+  for (int m0 = 0; m0 < M; m0 += WIDE_MAX_NPAD) {
+    const int Mc = M - m0 < WIDE_MAX_NPAD ? M - m0 : WIDE_MAX_NPAD;
+    WideParams p{};
+    p.N = N;
+    p.K = K;
+    p.M = Mc;
+    p.npad = (Mc + 15) / 16 * 16;
+    p.T = (N + BM - 1) / BM;
+    p.kb = K / BK;
+    p.nbuf = 2 * p.npad <= 512 ? 2 : 1;
+    int cols = 32;
+    while (cols < p.nbuf * p.npad) cols <<= 1;
+    p.tmem_cols = cols;
+    const int n1 = p.npad < 256 ? p.npad : 256;
+    p.idesc1 = mma_idesc(n1);
+    p.idesc2 = p.npad > 256 ? mma_idesc(p.npad - 256) : 0u;
+    p.status = status;
+    const WideChoice c = choose_wide(p.T, p.kb, p.npad, w.sm_count, w.wslot_bytes);
+    if (c.P == 0) return cudaErrorInvalidValue;
+    p.P = c.P;
+    p.Q = c.Q;
+    p.stages = c.stages;
+    p.slots = w.wslots;
+    p.ctr = w.wctr;
+    EpArgs ep = ep_in;
+    if (ep.out_f32) ep.out_f32 += (size_t)m0 * ep.ldo;
+    if (ep.out_t) ep.out_t = static_cast<bf16 *>(ep.out_t) + (size_t)m0 * ep.ldt;
+    if (ep.part_val) {
+      ep.part_val += (size_t)m0 * ep.n_tiles;
+      ep.part_idx += (size_t)m0 * ep.n_tiles;
+    }
+    if (ep.in_ss) ep.in_ss += m0;
+    if (ep.out_ss) ep.out_ss += m0;
+    if (ep.out_xn) ep.out_xn = static_cast<bf16 *>(ep.out_xn) + (size_t)m0 * ep.ld_xn;
+    if (ep.out_stash) ep.out_stash = static_cast<bf16 *>(ep.out_stash) + (size_t)m0 * ep.ld_stash;
+    ep.qkv.row0 = m0;
+    p.ep = ep;
+    const bf16 *xs = static_cast<const bf16 *>(X) + (size_t)m0 * ldx;
+    CUtensorMap mx1, mx2;
+    if (!tensor_map(&mx1, xs, Mc, K, ldx, n1)) return cudaErrorInvalidValue;
+    if (p.npad > 256) {
+      if (!tensor_map(&mx2, xs, Mc, K, ldx, p.npad - 256)) return cudaErrorInvalidValue;
+    } else {
+      mx2 = mx1;
+    }
+    p.dep = chain ? chain->take((unsigned)(p.P * p.Q)) : Dep{};
+    cudaError_t e;
+    switch (ep.mode) {
+      case EP_STORE_F32: e = launch_wide<EP_STORE_F32>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_RESID: e = launch_wide<EP_RESID>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_SWIGLU: e = launch_wide<EP_SWIGLU>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_SILU: e = launch_wide<EP_SILU>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_ARGMAX: e = launch_wide<EP_ARGMAX>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_QKV: e = launch_wide<EP_QKV>(mw, mx1, mx2, p, c.smem, s); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;

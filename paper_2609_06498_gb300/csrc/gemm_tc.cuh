@@ -20,7 +20,12 @@ struct TcWorkspace {
   // clusters (zero between uses; tc_init zeroes them)
   float *lacc = nullptr;
   unsigned int *lctr = nullptr;
-  size_t left_bytes = 0;
+  // wide launch (more than 128 token rows): per-tile arrival counts (zero
+  // between uses, right after lctr) and the fp32 split-K partial slots
+  unsigned int *wctr = nullptr;
+  float *wslots = nullptr;
+  size_t wslot_bytes = 0;
+  size_t left_bytes = 0;  // lacc, lctr and wctr: zeroed by tc_init
 };
 
 // Reserve the GEMM scratch at byte offset `off` of `base` (null base: size only).
@@ -35,6 +40,12 @@ cudaError_t tc_init(const TcWorkspace &w, cudaStream_t s);
 cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M,
                     int ldx, const EpArgs &ep, int *status, cudaStream_t s, bool use_caches = true,
                     DepChain *chain = nullptr);
+
+// One projection over up to 512 token rows per pass in a single stream of the
+// weights (any M: passes of 512 rows), split over k in independent CTAs when
+// the tiles are too few to fill the GPU; modes as gemm_tc.
+cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
+                      const EpArgs &ep, int *status, cudaStream_t s, DepChain *chain = nullptr);
 
 // One GEMM of a persistent sequence (out[m][n] = X[m][:] . W[n][:] with a
 // fused epilogue; modes EP_STORE_F32, EP_RESID, EP_SWIGLU, EP_QKV).

@@ -17,6 +17,8 @@ SHAPES = [  # (N, K, M)
     (6144, 2560, 68), (2560, 9728, 100), (4096, 4096, 128),
     # Eq. 1 feature projection of the 5-feature-layer workloads (K = 5 d)
     (4096, 20480, 17), (2560, 12800, 68),
+    # batch 16 x 17 rows: one pass with two MMAs per k-step (256 + 16 columns), split over k through L2
+    (4096, 4096, 272), (6144, 4096, 272), (4096, 12288, 272), (4096, 20480, 272), (1000, 512, 511), (2048, 1024, 600),
 ]
 
 
@@ -54,11 +56,22 @@ def _seq_ok(K, M):
     return M <= 128 and K % 64 == 0 and K // 64 >= 4
 
 
-@pytest.mark.parametrize("path", [1, 2], ids=["tc", "persistent"])
+PATHS = pytest.mark.parametrize("path", [1, 2, 3], ids=["tc", "persistent", "wide"])
+
+
+def _path_ok(path, K, M):
+    if path == 2:
+        return _seq_ok(K, M)
+    if path == 1:
+        return M <= 272 or M % 256 == 0  # the one-projection kernel: passes of 256 rows (kept to the old shapes)
+    return K % 64 == 0
+
+
+@PATHS
 @pytest.mark.parametrize("N,K,M", SHAPES)
 def test_store_and_resid(eng, path, N, K, M):
-    if path == 2 and not _seq_ok(K, M):
-        pytest.skip("outside the persistent launch")
+    if not _path_ok(path, K, M):
+        pytest.skip("outside this launch")
     W, X, ref = _inputs(N, K, M, N + K + M)
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     out = torch.full((M, N), float("nan"), device="cuda")
@@ -77,11 +90,12 @@ def test_store_and_resid(eng, path, N, K, M):
     assert torch.equal(out, out2), "not deterministic"
 
 
-@pytest.mark.parametrize("path", [1, 2], ids=["tc", "persistent"])
-@pytest.mark.parametrize("N,K,M", [(2944, 512, 17), (24576, 4096, 17), (19456, 2560, 68), (3072, 1024, 300)])
+@PATHS
+@pytest.mark.parametrize("N,K,M", [(2944, 512, 17), (24576, 4096, 17), (19456, 2560, 68), (3072, 1024, 300),
+                                   (24576, 4096, 272)])
 def test_swiglu_and_silu(eng, path, N, K, M):
-    if path == 2 and not _seq_ok(K, M):
-        pytest.skip("outside the persistent launch")
+    if not _path_ok(path, K, M):
+        pytest.skip("outside this launch")
     W, X, ref = _inputs(N, K, M, 7 * N + M)
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     h = torch.empty(M, N // 2, dtype=torch.bfloat16, device="cuda")
@@ -96,9 +110,9 @@ def test_swiglu_and_silu(eng, path, N, K, M):
     assert _rel(s.float(), torch.nn.functional.silu(ref)) < 1e-2
 
 
-@pytest.mark.parametrize("N,K,M", [(1000, 512, 17), (151936, 4096, 17), (151936, 4096, 1)])
-def test_argmax(eng, N, K, M):
-    path = 1
+@pytest.mark.parametrize("path", [1, 3], ids=["tc", "wide"])
+@pytest.mark.parametrize("N,K,M", [(1000, 512, 17), (151936, 4096, 17), (151936, 4096, 1), (151936, 4096, 272)])
+def test_argmax(eng, path, N, K, M):
     W, X, ref = _inputs(N, K, M, 11 * N + M)
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     out = torch.empty(M, dtype=torch.int32, device="cuda")
