@@ -9,4 +9,5 @@ each function follows.
 """
 from .dflow_oracle import (  # noqa: F401
     Oracle, State, RoundOut, rmsnorm, layernorm, silu, rope, attend, argmax_rows, top2_gap,
+    log_softmax, gumbel_argmax, speculative_sample,
 )

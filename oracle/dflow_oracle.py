@@ -16,7 +16,9 @@ in the order the paper states the method:
   * Sec. 4.2, Eq. 4 -- reject-conditioned MLP  [beta; gamma] = MLP([E(b); E(y_{a+1}); h])
   * Sec. 4.2, Eq. 5 -- x = E_mask + beta * LN(h) + gamma at valid carried slots,
                       E_mask elsewhere, masks only when nothing is carried
-  * Sec. 5.2        -- the autoregressive baseline (one greedy target step)
+  * Sec. 5.2        -- the autoregressive baseline (one greedy target step), and
+                      T = 1 verification by speculative sampling (a reading:
+                      the paper reports T = 1 results without printing the rule)
 
 Readings of points the paper leaves open (all shared with the CUDA path by
 specification, not by code):
@@ -118,6 +120,44 @@ def top2_gap(logits):
     """top-1 minus top-2 logit per row (how safely the argmax is decided)."""
     part = np.sort(np.asarray(logits, F), axis=-1)
     return part[..., -1] - part[..., -2]
+
+
+def log_softmax(z):
+    """log of the softmax of the last axis (temperature 1), in float64."""
+    z = np.asarray(z, F)
+    m = z.max(axis=-1, keepdims=True)
+    return z - m - np.log(np.exp(z - m).sum(axis=-1, keepdims=True))
+
+
+def gumbel_argmax(logw, g):
+    """A sample of the distribution proportional to exp(logw) by the Gumbel-max
+    rule: argmax_v (logw_v + g_v) with g_v standard Gumbel; -inf never wins."""
+    return int(np.argmax(np.asarray(logw, F) + np.asarray(g, F)))
+
+
+def speculative_sample(block, p_logits, q_logits, ua, gr):
+    """T = 1 verification of one draft block by speculative sampling (the reading
+    of Sec. 5.2's T = 1 rows: the paper does not print its rule; this is the
+    standard rule for proposals drawn from a known distribution).
+
+    p_i = softmax(p_logits[i - 1]) is the target's distribution for offset i
+    (verify row i - 1), q_i = softmax(q_logits[i]) the drafter's for the
+    proposal block[i], i = 1..B.  Proposal i is accepted when ua[i] <
+    p_i(y_i) / q_i(y_i); at the first rejection the token of offset i is drawn
+    from max(0, p_i - q_i) normalised; after B acceptances the bonus is drawn
+    from p_{B+1}.  gr[i - 1] is the Gumbel noise of offset i's draw.
+    Returns (a, token committed after the a accepted proposals)."""
+    B = len(block) - 1
+    for i in range(1, B + 1):
+        lp, lq = log_softmax(p_logits[i - 1]), log_softmax(q_logits[i])
+        y = int(block[i])
+        if np.log(ua[i]) < lp[y] - lq[y]:
+            continue
+        r = np.exp(lp) - np.exp(lq)
+        with np.errstate(divide="ignore"):
+            logr = np.where(r > 0, np.log(np.where(r > 0, r, 1.0)), -np.inf)
+        return i - 1, gumbel_argmax(logr, gr[i - 1])
+    return B, gumbel_argmax(log_softmax(p_logits[B]), gr[B])
 
 
 # ---------------------------------------------------------------------------
@@ -313,8 +353,9 @@ class Oracle:
 
     # -- Eq. 2: one-shot block drafting -------------------------------------
 
-    def draft_block(self, st: State, b: int, x: Optional[np.ndarray] = None):
-        """Drafter forward over the B+1 block rows; argmax of rows 1..B.
+    def draft_block(self, st: State, b: int, x: Optional[np.ndarray] = None, gd: Optional[np.ndarray] = None):
+        """Drafter forward over the B+1 block rows; argmax of rows 1..B, or with
+        gd (Gumbel noise [B+1][V]) a T = 1 sample of each row's distribution.
 
         Keys/values of draft layer l are [context K/V at 0..n-2 ; block rows],
         all visible to every block row.  Returns (block tokens, logits, inputs).
@@ -335,7 +376,8 @@ class Oracle:
         logits = self.lm_logits(x, "d.final_norm")
         block = np.empty(c.rows, np.int32)
         block[0] = st.tokens[b, n - 1]
-        block[1:] = argmax_rows(logits[1:])
+        block[1:] = argmax_rows(logits[1:]) if gd is None else [gumbel_argmax(logits[i], gd[i])
+                                                                 for i in range(1, c.rows)]
         return block, logits, x0
 
     # -- Eq. 3: verification ---------------------------------------------------
@@ -415,6 +457,40 @@ class Oracle:
             a, comm = self.accept_commit(st, b, blk, g, None if forced is None else forced[b])
             self.carry_hidden(st, b, blk, feats, a, relay)
             out.block[b], out.g[b], out.feats[b] = blk, g, feats
+            out.accept[b], out.committed[b] = a, comm
+        return out
+
+    # -- one round with T = 1 sampling verification (Sec. 5.2, Table 1 T = 1) --
+
+    def round_sampled(self, st: State, noise: Callable[[int], Dict[str, np.ndarray]],
+                      relay: bool = True) -> RoundOut:
+        """draft (T = 1 samples) -> verify -> speculative sampling -> commit -> carry.
+
+        noise(b) gives sequence b's draws for this round (synth.sampling_noise:
+        gd, ua, gr).  The relay and the carry are those of the greedy round: the
+        boundary tokens are the committed last token and the first rejected
+        proposal."""
+        c = self.cfg
+        bs, R, V = c.batch, c.rows, c.vocab
+        out = RoundOut(block=np.zeros((bs, R), np.int32), draft_logits=np.zeros((bs, R, V)),
+                       draft_x=np.zeros((bs, R, c.d)), g=np.zeros((bs, R), np.int32),
+                       verify_logits=np.zeros((bs, R, V)), feats=np.zeros((bs, R, c.d)),
+                       accept=np.zeros(bs, np.int32), committed=np.full((bs, R), -1, np.int32),
+                       n_before=st.seq_len.copy())
+        for b in range(bs):
+            if not st.active[b]:
+                continue
+            if not relay:
+                st.n_carry[b] = 0
+            nz = noise(b)
+            blk, out.draft_logits[b], out.draft_x[b] = self.draft_block(st, b, gd=nz["gd"])
+            g, out.verify_logits[b], feats = self.verify_block(st, b, blk)
+            a, tok = speculative_sample(blk, out.verify_logits[b], out.draft_logits[b], nz["ua"], nz["gr"])
+            gs = np.array(g, copy=True)
+            gs[a] = tok
+            a, comm = self.accept_commit(st, b, blk, gs, a)
+            self.carry_hidden(st, b, blk, feats, a, relay)
+            out.block[b], out.g[b], out.feats[b] = blk, gs, feats
             out.accept[b], out.committed[b] = a, comm
         return out
 

@@ -369,3 +369,55 @@ def block_tokens(cfg: ModelConfig, anchors: np.ndarray, seed: int = SEED_STATE) 
     out = uniform_ints(seed, "st.block", cfg.batch * cfg.rows, 0, cfg.vocab).reshape(cfg.batch, cfg.rows)
     out[:, 0] = anchors
     return out
+
+
+# --------------------------------------------------------------------------
+# random draws of T = 1 sampling verification: a counter-based SplitMix64
+# stream per (seed, sequence, round, row, purpose), indexed by token id.  The
+# draws are 24-bit uniforms in (0, 1), exactly representable in fp32, so a
+# float32 and a float64 consumer see the same number.
+# --------------------------------------------------------------------------
+
+NOISE_DRAFT, NOISE_ACCEPT, NOISE_RESAMPLE = 0, 1, 2
+SEED_SAMPLING = 4
+
+
+def noise_key(seed: int, seq: int, rnd: int, row: int, purpose: int) -> int:
+    """Key of one (sequence, round, row, purpose) stream."""
+    return splitmix64(seed ^ splitmix64((seq << 48) ^ (rnd << 24) ^ (row << 8) ^ purpose))
+
+
+def _splitmix64_np(x: np.ndarray) -> np.ndarray:
+    """SplitMix64 finaliser on uint64 arrays (wrap-around arithmetic)."""
+    with np.errstate(over="ignore"):
+        z = x + np.uint64(0x9E3779B97F4A7C15)
+        z = (z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)
+        z = (z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)
+        return z ^ (z >> np.uint64(31))
+
+
+def noise_uniform(key: int, n: int) -> np.ndarray:
+    """Uniforms u_v = (top 24 bits of splitmix64(key ^ v) + 0.5) / 2^24, v = 0..n-1 (float64)."""
+    v = np.arange(n, dtype=np.uint64) ^ np.uint64(key)
+    z = _splitmix64_np(v)
+    return ((z >> np.uint64(40)).astype(np.float64) + 0.5) / float(1 << 24)
+
+
+def sampling_noise(cfg: ModelConfig, seq: int, rnd: int, seed: int = SEED_SAMPLING) -> Dict[str, np.ndarray]:
+    """The draws one T = 1 round of sequence `seq` consumes.
+
+    gd [R][V]: Gumbel noise -log(-log u) of the drafter's sample at rows 1..B (row 0 unused)
+    ua [R]:    uniform of the acceptance test of the proposal in row i (i = 1..B; row 0 unused)
+    gr [R][V]: Gumbel noise of the token sampled for offset i = 1..B+1 (index i - 1):
+               the residual after a rejection at i, or the bonus after B acceptances
+    """
+    R, V = cfg.rows, cfg.vocab
+    gd = np.zeros((R, V))
+    gr = np.zeros((R, V))
+    ua = np.zeros(R)
+    for i in range(1, R):
+        gd[i] = -np.log(-np.log(noise_uniform(noise_key(seed, seq, rnd, i, NOISE_DRAFT), V)))
+        ua[i] = noise_uniform(noise_key(seed, seq, rnd, i, NOISE_ACCEPT), 1)[0]
+    for i in range(1, R + 1):
+        gr[i - 1] = -np.log(-np.log(noise_uniform(noise_key(seed, seq, rnd, i, NOISE_RESAMPLE), V)))
+    return {"gd": gd, "ua": ua, "gr": gr}
