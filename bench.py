@@ -30,6 +30,7 @@ import synth  # noqa: E402
 
 METRIC = "draft+verify round latency & committed tokens/s, Qwen3-8B shape; % HBM roofline"
 DEFAULT_CONFIG = "qwen3_8b_b1"
+T1_SEED = 4  # seed of the T = 1 leg's draws
 
 
 def parse():
@@ -590,6 +591,26 @@ def main():
                       "delta_frac": round((on - off) / off, 4),
                       "paper": "0.51 ms, 1.2 % of a DFlash round (Sec. 5.3; A800, model not stated)"}
 
+    # ---- T = 1 rounds (Sec. 5.2, Table 1 T = 1 rows): K speculative-sampling rounds from the same state
+    t1 = None
+    if rank == 0 and world == 1:
+        wl.restore()
+        n_start = st.seq_len.clone()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for k in range(K):
+            eng.round_sampled(st, T1_SEED, Wm + k, relay=relay, out=(wl.acc, wl.comm))
+        s1.record(stream)
+        torch.cuda.synchronize()
+        code = eng.read_status(st)
+        assert code == 0, f"device status {code} set during the T = 1 leg"
+        t1_ms = s0.elapsed_time(s1) / K
+        grown = float((st.seq_len - n_start).float().mean())
+        t1 = {"ms_per_round": round(t1_ms, 4), "greedy_ms_per_round": round(total_local / K, 4),
+              "delta_ms": round(t1_ms - total_local / K, 4), "mean_accept": round(grown / K - 1, 3),
+              "note": "random-init drafter and target: the acceptance is what the draws give; "
+                      "a round streams the same weights whatever it accepts"}
+
     # ---- autoregressive baseline (Sec. 5.2, Table 2 "Baseline"): K plain greedy steps of the
     # target from the same state, one committed token per sequence per step
     ar = None
@@ -654,6 +675,7 @@ def main():
         "step_split_ms": step_split,
         "relay_overhead": relay_cost,
         "ar_baseline": ar,
+        "t1_sampling": t1,
         "gpu_launches": int(launches),
         "e2e": e2e,
         "clocks": clocks.summary(),

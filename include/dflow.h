@@ -16,6 +16,8 @@
  *                       (alignment: keep the shifted verifier states of the
  *                       rejected suffix and the two boundary tokens).
  *   dflow_round         the four calls above in order, for the whole batch.
+ *   dflow_round_sampled one round at temperature 1 (Sec. 5.2): sampled
+ *                       proposals, speculative-sampling acceptance.
  *
  * Conventions shared by every call
  *   - Pointers in dflow_weights and dflow_state and every output pointer are
@@ -198,6 +200,33 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
                          int32_t *accept_len, int32_t *committed, int32_t relay,
                          void *stream);
 
+/* One full round at temperature 1 (Sec. 5.2, Table 1 T = 1 rows).  The paper
+ * does not print its T = 1 rule; this round applies standard speculative
+ * sampling per block position:
+ *   - block row i = 1..B holds a sample y_i of q_i = softmax(drafter logits
+ *     of row i);
+ *   - proposal i is accepted while u_i < p_i(y_i) / q_i(y_i), p_i =
+ *     softmax(target logits of verify row i-1);
+ *   - the token after the a accepted proposals is drawn from max(0, p_i -
+ *     q_i) normalised (i = a+1 <= B), or from p_{B+1} when a = B.
+ * Commit, carry and relay follow dflow_round with that token as the bonus
+ * and the first rejected proposal as boundary token.  Each draw is a
+ * Gumbel-max sample argmax_v(log w_v - log(-log u_v)); u_v comes from a
+ * SplitMix64 counter stream keyed by (seed, sequence index b, round_index,
+ * block row, purpose 0 = proposal / 1 = acceptance test / 2 = committed
+ * token), u_v = (2 (splitmix64(key ^ v) >> 41) + 1) / 2^24 with
+ * key = splitmix64(seed ^ splitmix64(b << 48 ^ round_index << 24 ^
+ * row << 8 ^ purpose)); the acceptance uniform of row i is v = 0 of its stream.
+ * The caller advances round_index (0 <= round_index < 2^24) between rounds.
+ * accept_len, committed: as for dflow_accept_commit.  draft_logits,
+ * verify_logits: optional device fp32 [batch][B+1][vocab]; where non-null the
+ * round writes that stage's logits there (and reads them back from there),
+ * else it uses workspace memory.  bf16 and fp32 handles; the round streams
+ * the LM head once per stage, as the greedy round does. */
+dflow_status dflow_round_sampled(dflow_handle *h, dflow_state *st, uint64_t seed, int32_t round_index,
+                                 int32_t *accept_len, int32_t *committed, int32_t relay,
+                                 float *draft_logits, float *verify_logits, void *stream);
+
 /* Sec. 5.2, Table 2 "Baseline": one step of plain autoregressive greedy
  * decoding of the target, for every active sequence: the last committed token
  * (position n-1) runs through the target against the cached K/V (its K/V are
@@ -235,9 +264,10 @@ dflow_status dflow_profile_enable(dflow_handle *h, int32_t enable);
 /* Test hook: one projection out[m][n] = sum_k X[m][k] W[n][k] through the
  * library's GEMM kernels (path 0: CUDA-core kernel of fp32 handles; bf16
  * handles: path 1 the tcgen05 kernel of one projection, path 2 the persistent
- * tcgen05 launch the round uses for up to 128 rows (modes 0-3, K a multiple of
- * 64 and at least 256), path 3 the one-pass tcgen05 launch the round uses above
- * 128 rows; else DFLOW_ERR_UNSUPPORTED), with the epilogue `mode`: 0 store fp32 out[M][ldo];
+ * tcgen05 launch the round uses for 16 to 128 rows (modes 0-3, K a multiple of
+ * 64 and at least 256; fewer rows are refused before any launch), path 3 the
+ * one-pass tcgen05 launch the round uses above 128 rows for shapes it suits;
+ * else DFLOW_ERR_UNSUPPORTED), with the epilogue `mode`: 0 store fp32 out[M][ldo];
  * 1 add into fp32 out[M][ldo]; 2 SwiGLU of 128-row [64 gate | 64 up] groups
  * into model-dtype out[M][ldo] (N/2 features); 3 SiLU into model-dtype out;
  * 4 greedy argmax over n into int32 out[M] (M <= max_batch * max(B+1, 64)).

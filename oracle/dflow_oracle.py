@@ -154,6 +154,8 @@ def speculative_sample(block, p_logits, q_logits, ua, gr):
         if np.log(ua[i]) < lp[y] - lq[y]:
             continue
         r = np.exp(lp) - np.exp(lq)
+        if not (r > 0).any():  # only through rounding (a rejection implies p_i(v) > q_i(v) somewhere): draw from p_i
+            return i - 1, gumbel_argmax(lp, gr[i - 1])
         with np.errstate(divide="ignore"):
             logr = np.where(r > 0, np.log(np.where(r > 0, r, 1.0)), -np.inf)
         return i - 1, gumbel_argmax(logr, gr[i - 1])

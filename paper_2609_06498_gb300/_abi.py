@@ -67,6 +67,8 @@ _SIGS = {
     "dflow_carry_hidden": ([_P, ctypes.POINTER(State), _P, _P, _P, _P], ctypes.c_int),
     "dflow_decode_step": ([_P, ctypes.POINTER(State), _P, ctypes.c_int32, _P], ctypes.c_int),
     "dflow_round": ([_P, ctypes.POINTER(State), _P, _P, _P, ctypes.c_int32, _P], ctypes.c_int),
+    "dflow_round_sampled": ([_P, ctypes.POINTER(State), ctypes.c_uint64, ctypes.c_int32, _P, _P, ctypes.c_int32, _P,
+                             _P, _P], ctypes.c_int),
     "dflow_read_status": ([_P, ctypes.POINTER(State), c_i32p, _P], ctypes.c_int),
     "dflow_profile_enable": ([_P, ctypes.c_int32], ctypes.c_int),
     "dflow_profile_read": ([_P, ctypes.POINTER(KernelProfile)], ctypes.c_int),

@@ -12,6 +12,7 @@
 
 #include "dflow_internal.cuh"
 #include "gemm_tc.cuh"
+#include "sample.cuh"
 
 using namespace dflow;
 
@@ -462,6 +463,8 @@ struct dflow_handle {
   float2 *rope;
   void *xn, *q, *bk, *bv, *ao, *mlp, *stash, *feats, *relay_u, *relay_h;
   int *pos, *wr, *pos2, *wr2, *am_idx, *blk, *g, *gd, *acc, *comm, *plen, *kvlen, *zeros;
+  float *qlog, *plog;  // T = 1 round: drafter and target logits [rows_round][vocab]
+  SampWs samp;
   TcWorkspace tcw;
   DepChain dep;  // completion counters between consecutive tensor-core launches
   // measurement
@@ -541,6 +544,16 @@ size_t layout(dflow_handle *h, char *base) {
   h->plen = (int *)take((size_t)c.max_batch * 4);
   h->kvlen = (int *)take((size_t)c.max_batch * 4);
   h->zeros = (int *)take((size_t)c.max_batch * 4);
+  const size_t rr = h->rows_round;
+  h->qlog = (float *)take(rr * D.vocab * 4);
+  h->plog = (float *)take(rr * D.vocab * 4);
+  h->samp.nch = samp_chunks(D.vocab);
+  h->samp.part = (float2 *)take(rr * h->samp.nch * 8);
+  h->samp.gv = (float *)take(rr * h->samp.nch * 4);
+  h->samp.gi = (int *)take(rr * h->samp.nch * 4);
+  h->samp.lse_q = (float *)take(rr * 4);
+  h->samp.lse_p = (float *)take(rr * 4);
+  h->samp.a = (int *)take((size_t)c.max_batch * 4);
   h->rope = (float2 *)take((size_t)c.max_ctx * (D.hd / 2) * 8);
   h->dep.dev = (unsigned int *)take(kDepSlots * sizeof(unsigned int));
   const int max_n = std::max(std::max(D.vocab, 2 * D.inter), std::max(h->gld, D.d));
@@ -612,8 +625,10 @@ cudaError_t gemm(const Call &k, const void *W, int N, int K, const void *X, int 
     return gemm_seq(h->tcw, 1, &sp, M, k.status_w, k.s, &h->dep);
   }
   if (!tc_supports(N, K, M, ldx, ep)) return cudaErrorInvalidValue;
-  // more rows than the persistent launch takes: one pass over the weights for up to 512 rows
-  if (M > 128) return gemm_wide(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, &h->dep);
+  // more rows than the persistent launch takes: one pass over the weights for up
+  // to 512 rows where its schedule suits the shape, else 128-row tiles
+  if (M > 128 && gemm_wide_suits(h->tcw, N, K, M))
+    return gemm_wide(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, &h->dep);
   return gemm_tc(h->tcw, W, N, K, X, M, ldx, ep, k.status_w, k.s, true, &h->dep);
 }
 
@@ -799,7 +814,8 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
   return cudaSuccess;
 }
 
-// final RMSNorm -> LM head -> greedy token per row (and fp32 logits when asked)
+// final RMSNorm -> LM head -> greedy token per row (g non-null) and fp32 logits
+// (logits non-null): one pass over the LM head per output asked for
 template <typename T>
 cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *norm, int *g,
                            float *logits) {
@@ -812,9 +828,12 @@ cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *
   ep.part_idx = h->am_idx;
   ep.n_tiles = h->vocab_tiles;
   if (h->fused) ep = in_norm(ep, h);
-  if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
-  KL(klaunch(k_argmax_reduce, (rows + 7) / 8, 256, 0, k.s, h->am_val, h->am_idx, h->vocab_tiles, rows, g, k.status));
-  if ((e = cudaGetLastError())) return e;
+  if (g) {
+    if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
+    KL(klaunch(k_argmax_reduce, (rows + 7) / 8, 256, 0, k.s, h->am_val, h->am_idx, h->vocab_tiles, rows, g,
+               k.status));
+    if ((e = cudaGetLastError())) return e;
+  }
   if (logits) {
     EpArgs el = ep_f32(logits, D.vocab);
     if (h->fused) el = in_norm(el, h);
@@ -960,7 +979,8 @@ Dims round_dims(const dflow_handle *h) {
 }
 
 template <typename T>
-dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float *logits = nullptr) {
+dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float *logits = nullptr,
+                      const SampRound *sr = nullptr) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R, B = D.B;
@@ -995,6 +1015,18 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float
   const int splits = pick_splits(h, batch, rows);
   CK(stack_forward<T>(k, D, batch, h->dl.data(), h->cfg.draft_layers, static_cast<T *>(st->draft_kv), st, 0, splits,
                       h->w.draft_final_norm));
+  if (sr != nullptr) {
+    // T = 1: logits only, then a Gumbel-max sample per block row
+    CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, nullptr, logits));
+    int n = 0;
+    const cudaError_t e = samp_draft(logits, D.vocab, D.R, batch, *sr, h->samp, st->tokens, st->seq_len, st->active,
+                                     h->cfg.max_ctx, blk, k.status, k.s, &n);
+    h->n_launch += n;
+    h->dep.brk();
+    CK(e);
+    CK(cudaGetLastError());
+    return DFLOW_OK;
+  }
   CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, logits));
   KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
                                                    D.R, blk, k.status));
@@ -1039,6 +1071,28 @@ dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void
                                                D.d, D.B, relay, k.status));
   CK(cudaGetLastError());
   return DFLOW_OK;
+}
+
+// Sec. 5.2, T = 1: draft (samples) -> verify (logits) -> speculative sampling
+// (acceptance length and the token after it) -> Eq. 3 commit with that
+// acceptance forced -> carry
+template <typename T>
+dflow_status do_round_sampled(const Call &k, dflow_state *st, SampRound sr, int *acc, int *comm, int relay,
+                              float *qlog, float *plog) {
+  dflow_handle *h = k.h;
+  const int batch = st->batch, R = h->R;
+  dflow_status r;
+  if ((r = do_draft<T>(k, st, h->blk, relay, qlog, &sr))) return r;
+  if ((r = do_verify<T>(k, st, h->blk, nullptr, h->feats, plog))) return r;
+  int n = 0;
+  const cudaError_t e = samp_verify(plog, qlog, h->D.vocab, R, batch, sr, h->samp, h->blk, st->active, h->g,
+                                    k.status, k.s, &n);
+  h->n_launch += n;
+  h->dep.brk();
+  CK(e);
+  CK(cudaGetLastError());
+  if ((r = do_accept(k, st, h->blk, h->g, h->samp.a, acc, comm))) return r;
+  return do_carry<T>(k, st, h->blk, h->feats, acc, relay);
 }
 
 // Sec. 5.2 baseline: one greedy step of the target alone.  The step runs on the
@@ -1352,6 +1406,20 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
   if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
   if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
   return finish(h, do_carry<float>(k, st, h->blk, h->feats, accept_len, relay));
+}
+
+dflow_status dflow_round_sampled(dflow_handle *h, dflow_state *st, uint64_t seed, int32_t round_index,
+                                 int32_t *accept_len, int32_t *committed, int32_t relay, float *draft_logits,
+                                 float *verify_logits, void *stream) {
+  dflow_status r = check_call(h, st);
+  if (r) return r;
+  if (!accept_len || !committed || round_index < 0 || round_index >= (1 << 24)) return DFLOW_ERR_INVALID_ARG;
+  Call k = make_call(h, st, stream);
+  if ((r = guard(k, st))) return finish(h, r);
+  const SampRound sr{seed, round_index};
+  float *q = draft_logits ? draft_logits : h->qlog, *p = verify_logits ? verify_logits : h->plog;
+  return finish(h, h->dtype == DFLOW_BF16 ? do_round_sampled<bf16>(k, st, sr, accept_len, committed, relay, q, p)
+                                          : do_round_sampled<float>(k, st, sr, accept_len, committed, relay, q, p));
 }
 
 dflow_status dflow_decode_step(dflow_handle *h, dflow_state *st, int32_t *token_out, int32_t draft_context,

@@ -1898,6 +1898,13 @@ cudaError_t launch_wide(const CUtensorMap &mw, const CUtensorMap &mx1, const CUt
 
 }  // namespace
 
+bool gemm_wide_suits(const TcWorkspace &w, int N, int K, int M) {
+  if (K < BK || K % BK) return false;
+  const int Mc = M < WIDE_MAX_NPAD ? M : WIDE_MAX_NPAD;
+  const WideChoice c = choose_wide((N + BM - 1) / BM, K / BK, (Mc + 15) / 16 * 16, w.sm_count, w.wslot_bytes);
+  return c.P == 1 || K / BK >= 128;
+}
+
 cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
                       const EpArgs &ep_in, int *status, cudaStream_t s, DepChain *chain) {
   if (N < 1 || K < BK || K % BK || M < 1 || ldx % 8 || (N + BM - 1) / BM > WIDE_MAX_TILES || w.wctr == nullptr)
@@ -2000,8 +2007,11 @@ static int seq_npad(int M) {
   return n == 112 ? 128 : n;
 }
 
+// From 16 rows: with a single row (16 padded columns, three owners without
+// columns) the launch faulted the GPU (gate/up 24576 x 4096 and O 4096 x 4096);
+// fewer than 16 rows take the row-tiled kernel.
 bool seq_supported(int M) {
-  return M >= 1 && seq_npad(M) <= SEQ_MAX_NPAD && encode_fn() != nullptr;
+  return M >= 16 && seq_npad(M) <= SEQ_MAX_NPAD && encode_fn() != nullptr;
 }
 
 // two Q/K/V epilogues build the same column table (positions and pool slots)

@@ -8,7 +8,7 @@ torch, and passes raw device pointers to the library.
 from __future__ import annotations
 
 import ctypes
-from typing import Dict, List, Optional, Sequence
+from typing import Dict, List, Optional, Sequence, Tuple
 
 import numpy as np
 import torch
@@ -257,6 +257,17 @@ class Engine:
         call("dflow_round", self.h, ctypes.byref(st.c),
              ctypes.c_void_p(forced.data_ptr() if forced is not None else 0), ctypes.c_void_p(acc.data_ptr()),
              ctypes.c_void_p(comm.data_ptr()), int(relay), self._stream())
+        return acc, comm
+
+    def round_sampled(self, st: DeviceState, seed: int, round_index: int, relay: bool = True, out=None,
+                      logits: Optional[Tuple[torch.Tensor, torch.Tensor]] = None):
+        """One T = 1 round (speculative sampling, see dflow_round_sampled); (accept_len, committed).
+        logits: optional fp32 (drafter, target) buffers [batch][B+1][vocab] that receive the round's logits."""
+        acc, comm = out if out is not None else (self._i32(st.batch), self._i32(st.batch, self.cfg.rows))
+        ql, pl = (0, 0) if logits is None else (logits[0].data_ptr(), logits[1].data_ptr())
+        call("dflow_round_sampled", self.h, ctypes.byref(st.c), ctypes.c_uint64(seed), int(round_index),
+             ctypes.c_void_p(acc.data_ptr()), ctypes.c_void_p(comm.data_ptr()), int(relay), ctypes.c_void_p(ql),
+             ctypes.c_void_p(pl), self._stream())
         return acc, comm
 
     def decode_step(self, st: DeviceState, draft_context: bool = False, out: Optional[torch.Tensor] = None):

@@ -374,8 +374,9 @@ def block_tokens(cfg: ModelConfig, anchors: np.ndarray, seed: int = SEED_STATE) 
 # --------------------------------------------------------------------------
 # random draws of T = 1 sampling verification: a counter-based SplitMix64
 # stream per (seed, sequence, round, row, purpose), indexed by token id.  The
-# draws are 24-bit uniforms in (0, 1), exactly representable in fp32, so a
-# float32 and a float64 consumer see the same number.
+# draws are odd multiples of 2^-24 in (0, 1), (2k + 1) / 2^24 with k the top 23
+# bits of the hash: exactly representable in fp32 (24 significant bits), so a
+# float32 and a float64 consumer see the same number, and never 0 or 1.
 # --------------------------------------------------------------------------
 
 NOISE_DRAFT, NOISE_ACCEPT, NOISE_RESAMPLE = 0, 1, 2
@@ -397,10 +398,10 @@ def _splitmix64_np(x: np.ndarray) -> np.ndarray:
 
 
 def noise_uniform(key: int, n: int) -> np.ndarray:
-    """Uniforms u_v = (top 24 bits of splitmix64(key ^ v) + 0.5) / 2^24, v = 0..n-1 (float64)."""
+    """Uniforms u_v = (2 (splitmix64(key ^ v) >> 41) + 1) / 2^24, v = 0..n-1 (float64)."""
     v = np.arange(n, dtype=np.uint64) ^ np.uint64(key)
     z = _splitmix64_np(v)
-    return ((z >> np.uint64(40)).astype(np.float64) + 0.5) / float(1 << 24)
+    return ((z >> np.uint64(41)).astype(np.float64) * 2.0 + 1.0) / float(1 << 24)
 
 
 def sampling_noise(cfg: ModelConfig, seq: int, rnd: int, seed: int = SEED_SAMPLING) -> Dict[str, np.ndarray]:

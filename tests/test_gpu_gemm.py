@@ -52,8 +52,8 @@ def _tol(K):
 
 
 def _seq_ok(K, M):
-    # the persistent launch (path 2) takes up to 128 rows and at least 4 k-blocks
-    return M <= 128 and K % 64 == 0 and K // 64 >= 4
+    # the persistent launch (path 2) takes 16 to 128 rows and at least 4 k-blocks
+    return 16 <= M <= 128 and K % 64 == 0 and K // 64 >= 4
 
 
 PATHS = pytest.mark.parametrize("path", [1, 2, 3], ids=["tc", "persistent", "wide"])
@@ -123,3 +123,17 @@ def test_argmax(eng, path, N, K, M):
     safe = (top2.values[:, 0] - top2.values[:, 1]) > 1e-3
     assert safe.any()
     assert torch.equal(out.long()[safe], top2.indices[:, 0][safe])
+
+
+def test_persistent_launch_refuses_fewer_than_16_rows(eng):
+    """Rows 1-15 never reach the persistent launch: the call is refused on the
+    host, before anything is launched (the round routes them to the row-tiled kernel)."""
+    from paper_2609_06498_gb300._abi import DFlowError
+    W, X, _ = _inputs(4096, 4096, 1, 3)
+    out = torch.zeros(1, 4096, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    with pytest.raises(DFlowError):
+        eng.debug_gemm(2, W, X, 0, out, st)
+    eng.debug_gemm(1, W, X, 0, out, st)  # the row-tiled kernel takes it
+    torch.cuda.synchronize()
+    assert int(st) == 0 and _rel(out, X.float() @ W.float().T) <= _tol(4096)

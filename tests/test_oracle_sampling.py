@@ -128,3 +128,6 @@ def test_sampling_noise_is_reproducible_and_uniform():
     u = np.exp(-np.exp(-a["gd"][1:].ravel()))  # back to the uniforms
     assert abs(u.mean() - 0.5) < 0.01 and scipy_stats.kstest(u, "uniform").pvalue > 1e-4
     assert ((a["ua"][1:] > 0) & (a["ua"][1:] < 1)).all()
+    raw = synth.noise_uniform(synth.noise_key(4, 0, 0, 1, synth.NOISE_DRAFT), 1 << 16)
+    assert (raw.astype(np.float32).astype(np.float64) == raw).all()  # the same value in fp32
+    assert raw.min() > 0 and raw.max() < 1 and np.isfinite(-np.log(-np.log(raw.astype(np.float32)))).all()
