@@ -27,7 +27,7 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {
 }
 
 constexpr int T5_ROWS = 128;     // query rows per CTA (MMA M)
-// key splits = cluster size S (8, or 4 when 8 would not fit in one wave); split s
+// key splits = cluster size S (8 when every 8-CTA cluster is resident at once, else 4); split s
 // takes pages s, s + S, ...
 constexpr float T5_TAU = 8.0f;   // rescale threshold, log2 units
 constexpr int T5_TMEM_COLS = 256;  // O: 128 columns, S: two buffers of 64

@@ -116,9 +116,9 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs 
   return cudaLaunchKernelEx(&cfg, k_attn_t5<BLOCK, S>, tm, tq, D, a, q_tma, status);
 }
 
-// eight key splits per (kv head, sequence, query group), or four when the
-// eight-CTA clusters would need a second wave and the four-CTA ones fit in one
-// (the per-CTA key loop is latency bound: one wave of twice the pages is shorter)
+// eight key splits per (kv head, sequence, query group) when every eight-CTA
+// cluster is resident at once, else four (a CTA's fixed costs, set-up, first
+// pages and the cluster merge, are paid by half as many CTAs)
 template <bool BLOCK>
 cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
                           cudaStream_t s, DepChain *chain) {
@@ -134,7 +134,9 @@ cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const
   }();
   if (forced == 4 && r4 >= 1) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
   if (forced == 8) return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
-  if (units > r8 && units <= r4) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
+  // 8 splits only when every cluster is resident at once; otherwise 4 (fewer,
+  // longer CTAs: at batch 16 and 1K-8K keys a launch took 0.64-0.70 of the time)
+  if (units > r8) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
   return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
 }
 
