@@ -131,3 +131,34 @@ def test_sampling_noise_is_reproducible_and_uniform():
     raw = synth.noise_uniform(synth.noise_key(4, 0, 0, 1, synth.NOISE_DRAFT), 1 << 16)
     assert (raw.astype(np.float32).astype(np.float64) == raw).all()  # the same value in fp32
     assert raw.min() > 0 and raw.max() < 1 and np.isfinite(-np.log(-np.log(raw.astype(np.float32)))).all()
+
+
+def test_draw_rows_follow_the_documented_convention():
+    """The token of offset i is drawn with gr[i - 1] (the bonus with gr[B]), the
+    proposal of row i with gd[i] and its test with ua[i]: hand cases where each
+    other row of draws would pick another token (no distribution test can see
+    which independent row is used; the GPU kernels key their draws the same way)."""
+    V, B, big = 4, 2, 50.0
+    p = np.zeros((B + 1, V))
+    p[:, 0] = -60.0  # the target never takes token 0
+    q = np.full((B + 1, V), -60.0)
+    q[:, 0] = 0.0  # the drafter always proposes token 0: rejected at offset 1
+    gr = np.zeros((B + 1, V))
+    gr[0, 2] = big  # offset 1's draw
+    gr[1, 3] = big
+    gr[2, 1] = big
+    a, tok = speculative_sample([7, 0, 0], p, q, np.full(B + 1, 0.5), gr)
+    assert (a, tok) == (0, 2)
+    # all accepted (q = p): the bonus comes from p_{B+1} with gr[B]
+    q2 = np.vstack([np.zeros(V), p[:B]])
+    a, tok = speculative_sample([7, 1, 1], p, q2, np.full(B + 1, 0.5), gr)
+    assert (a, tok) == (B, 1)
+    # the acceptance test of row i reads ua[i]: u = 1 - 1e-9 rejects wherever p/q < 1
+    p3 = np.log(np.array([[0.5, 0.5, 1e-9, 1e-9]] * (B + 1)))
+    q3 = np.log(np.array([[0.9, 0.1, 1e-9, 1e-9]] * (B + 1)))
+    ua = np.array([0.0, 0.1, 1 - 1e-9])  # row 1 accepts (0.1 < 0.5/0.9), row 2 rejects
+    a, _ = speculative_sample([7, 0, 0], p3, q3, ua, gr)
+    assert a == 1
+    ua = np.array([0.0, 1 - 1e-9, 0.1])  # the other way round: row 1 rejects
+    a, _ = speculative_sample([7, 0, 0], p3, q3, ua, gr)
+    assert a == 0
