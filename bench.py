@@ -59,6 +59,11 @@ def parse():
     p.add_argument("--M", type=int, default=17)
     p.add_argument("--mode", type=int, default=4, help="0 fp32 store, 1 residual add, 2 SwiGLU, 3 SiLU, 4 argmax")
     p.add_argument("--reps", type=int, default=3)
+    p.add_argument("--path", type=int, default=1, choices=[1, 2, 3],
+                   help="with --kernel gemm: 1 row-tiled tcgen05 launch, 2 persistent launch (16-128 rows), "
+                        "3 one-pass launch (above 128 rows)")
+    p.add_argument("--cublas", action="store_true",
+                   help="with --kernel gemm: also time torch.matmul of the same bf16 tensors (for scale)")
     return p.parse_args()
 
 
@@ -351,19 +356,32 @@ def run_kernel_gemm(args):
         out = torch.zeros(M, N // 2 if mode == 2 else N, dtype=torch.bfloat16, device="cuda")
     else:
         out = torch.zeros(M, dtype=torch.int32, device="cuda")
-    eng.debug_gemm(1, W, X, mode, out, st)  # warm-up (tensor maps, attributes)
+    for _ in range(3):  # warm-up (tensor maps, attributes)
+        eng.debug_gemm(args.path, W, X, mode, out, st)
     torch.cuda.synchronize()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
     evs[0].record()
     for r in range(args.reps):
-        eng.debug_gemm(1, W, X, mode, out, st)
+        eng.debug_gemm(args.path, W, X, mode, out, st)
         evs[r + 1].record()
     torch.cuda.synchronize()
     ms = [evs[r].elapsed_time(evs[r + 1]) for r in range(args.reps)]
     alg = 2.0 * N * K + 2.0 * M * K
-    print(json.dumps({"kernel": "gemm", "N": N, "K": K, "M": M, "mode": mode, "status": int(st),
-                      "ms": [round(x, 4) for x in ms], "alg_bytes": alg,
-                      "gbs_best": round(alg / min(ms) / 1e6, 1)}), flush=True)
+    rec = {"kernel": "gemm", "path": args.path, "N": N, "K": K, "M": M, "mode": mode, "status": int(st),
+           "ms": [round(x, 4) for x in ms], "ms_mean": round(float(np.mean(ms)), 4), "alg_bytes": alg,
+           "gbs_mean": round(alg / float(np.mean(ms)) / 1e6, 1), "tflops_mean": round(2.0 * N * K * M / float(np.mean(ms)) / 1e9, 1)}
+    if args.cublas:
+        for _ in range(3):
+            X @ W.T
+        torch.cuda.synchronize()
+        c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        c0.record()
+        for _ in range(args.reps):
+            X @ W.T
+        c1.record()
+        torch.cuda.synchronize()
+        rec["cublas_ms_mean"] = round(c0.elapsed_time(c1) / args.reps, 4)
+    print(json.dumps(rec), flush=True)
 
 
 # --------------------------------------------------------------------------
