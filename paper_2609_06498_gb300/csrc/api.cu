@@ -66,14 +66,38 @@ __global__ void k_guard(const int *tokens, const int *seq_len, const int *n_carr
   }
 }
 
-// rows of a round: row b*R+i at position n_b-1+i; writes allowed for active sequences
+// the state checks of k_guard, folded into k_rows_round
+struct GuardArgs {
+  const int *tokens = nullptr, *n_carry = nullptr, *boundary = nullptr;
+  int max_ctx = 0, vocab = 0, B = 0;
+  int *status = nullptr;  // null: no checks
+};
+
+// rows of a round: row b*R+i at position n_b-1+i; writes allowed for active
+// sequences.  With gd.status set, row 0 of each sequence also runs k_guard's
+// checks (the entry points whose first kernel this is launch no separate guard).
 __global__ void k_rows_round(int *pos, int *wr, int *kvlen, const int *seq_len, const int *active, int batch,
-                             int R, const int *status) {
+                             int R, const int *status, GuardArgs gd) {
   pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * R) return;
   const int b = r / R, i = r % R;
+  if (gd.status != nullptr && i == 0 && active[b]) {
+    const int n = seq_len[b];
+    if (n < 1 || n - 1 + R > gd.max_ctx) {
+      set_status(gd.status, DFLOW_ERR_CAPACITY);
+    } else {
+      const int anchor = gd.tokens[(size_t)b * gd.max_ctx + n - 1];
+      const int nc = gd.n_carry[b];
+      if (anchor < 0 || anchor >= gd.vocab || nc < 0 || nc > gd.B - 1) {
+        set_status(gd.status, DFLOW_ERR_BAD_STATE);
+      } else if (nc > 0) {
+        const int t0 = gd.boundary[2 * b], t1 = gd.boundary[2 * b + 1];
+        if (t0 < 0 || t0 >= gd.vocab || t1 < 0 || t1 >= gd.vocab) set_status(gd.status, DFLOW_ERR_BAD_STATE);
+      }
+    }
+  }
   const bool ok = active[b] != 0;
   pos[r] = ok ? seq_len[b] - 1 + i : 0;
   wr[r] = ok;
@@ -247,8 +271,16 @@ __global__ void k_stash(const float *__restrict__ x, T *__restrict__ stash, int 
 }
 
 // g[r] = argmax over the per-tile partials (ties: lowest token id)
+// the drafter's block tokens written straight from the argmax: row 0 of each
+// sequence is its anchor, rows 1..R-1 the predictions
+struct BlockOut {
+  int *blk = nullptr;
+  const int *tokens = nullptr, *seq_len = nullptr;
+  int max_ctx = 0, R = 1;
+};
+
 __global__ void k_argmax_reduce(const float *__restrict__ pv, const int *__restrict__ pi, int n_tiles,
-                                int rows, int *__restrict__ g, const int *status) {
+                                int rows, int *__restrict__ g, const int *status, BlockOut bo) {
   pdl_entry();
   if (*status) return;
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -257,7 +289,13 @@ __global__ void k_argmax_reduce(const float *__restrict__ pv, const int *__restr
   int idx = 0x7fffffff;
   for (int t = lane; t < n_tiles; t += 32) argmax_merge(v, idx, pv[(size_t)r * n_tiles + t], pi[(size_t)r * n_tiles + t]);
   warp_argmax(v, idx);
-  if (lane == 0) g[r] = idx;
+  if (lane == 0) {
+    g[r] = idx;
+    if (bo.blk != nullptr) {
+      const int b = r / bo.R, i = r % bo.R;
+      bo.blk[r] = i == 0 ? bo.tokens[(size_t)b * bo.max_ctx + bo.seq_len[b] - 1] : idx;
+    }
+  }
 }
 
 // relay MLP input (Eq. 4): u = [E(b); E(y_{a+1}); h_j] for each of the B slots
@@ -334,22 +372,14 @@ __global__ void k_draft_input(const T *__restrict__ E, const float *__restrict__
   }
 }
 
-__global__ void k_draft_out(const int *__restrict__ gd, const int *__restrict__ tokens,
-                            const int *__restrict__ seq_len, int max_ctx, int batch, int R,
-                            int *__restrict__ blk, const int *status) {
-  pdl_entry();
-  if (*status) return;
-  const int r = blockIdx.x * blockDim.x + threadIdx.x;
-  if (r >= batch * R) return;
-  const int b = r / R, i = r % R;
-  blk[r] = i == 0 ? tokens[(size_t)b * max_ctx + seq_len[b] - 1] : gd[r];
-}
-
 // Eq. 3: a, bonus, commit (one thread per sequence)
+// pos2 / wr2 (optional): the positions of the rows that join the drafter context
+// (what k_carry_rows computes from acc), filled here inside a round
 __global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
                          const int *__restrict__ forced, int *__restrict__ tokens,
                          int *__restrict__ seq_len, const int *__restrict__ active, int batch, int B,
-                         int max_ctx, int *__restrict__ acc, int *__restrict__ comm, int *status) {
+                         int max_ctx, int *__restrict__ acc, int *__restrict__ comm, int *status,
+                         int *__restrict__ pos2 = nullptr, int *__restrict__ wr2 = nullptr) {
   pdl_entry();
   if (*status) return;
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
@@ -360,6 +390,11 @@ __global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
   if (!active[b]) {
     acc[b] = -1;
     for (int i = 0; i < R; ++i) cb[i] = -1;
+    if (pos2 != nullptr)
+      for (int i = 0; i < R; ++i) {
+        pos2[(size_t)b * R + i] = 0;
+        wr2[(size_t)b * R + i] = 0;
+      }
     return;
   }
   int a = 0;
@@ -378,6 +413,11 @@ __global__ void k_accept(const int *__restrict__ blk, const int *__restrict__ g,
   }
   seq_len[b] = n + a + 1;
   acc[b] = a;
+  if (pos2 != nullptr)  // rows 0..a at positions n-1..n-1+a join the drafter context
+    for (int i = 0; i < R; ++i) {
+      pos2[(size_t)b * R + i] = i <= a ? n - 1 + i : 0;
+      wr2[(size_t)b * R + i] = i <= a ? 1 : 0;
+    }
 }
 
 // positions of the rows that join the drafter context after a commit
@@ -818,7 +858,7 @@ cudaError_t layer_forward(const Call &k, const Dims &D, int batch, const dflow_l
 // (logits non-null): one pass over the LM head per output asked for
 template <typename T>
 cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *norm, int *g,
-                           float *logits) {
+                           float *logits, BlockOut bo = BlockOut{}) {
   dflow_handle *h = k.h;
   cudaError_t e;
   if (!h->fused && (e = rmsnorm<T>(k, h->x, D.d, norm, h->xn, D.d, rows))) return e;
@@ -831,7 +871,7 @@ cudaError_t lm_head_argmax(const Call &k, const Dims &D, int rows, const float *
   if (g) {
     if ((e = gemm(k, h->w.lm_head, D.vocab, D.d, h->xn, rows, D.d, ep))) return e;
     KL(klaunch(k_argmax_reduce, (rows + 7) / 8, 256, 0, k.s, h->am_val, h->am_idx, h->vocab_tiles, rows, g,
-               k.status));
+               k.status, bo));
     if ((e = cudaGetLastError())) return e;
   }
   if (logits) {
@@ -972,6 +1012,19 @@ cudaError_t ctx_append(const Call &k, const Dims &D, int rows, const dflow_state
   return cudaSuccess;
 }
 
+// the round's device-side state checks, run by its first kernel (k_rows_round)
+GuardArgs guard_args(const Call &k, const dflow_state *st) {
+  GuardArgs g;
+  g.tokens = st->tokens;
+  g.n_carry = st->n_carry;
+  g.boundary = st->boundary;
+  g.max_ctx = k.h->cfg.max_ctx;
+  g.vocab = k.h->D.vocab;
+  g.B = k.h->D.B;
+  g.status = k.status_w;
+  return g;
+}
+
 Dims round_dims(const dflow_handle *h) {
   Dims D = h->D;
   D.R = h->R;
@@ -984,7 +1037,8 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R, B = D.B;
-  KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch, D.R, k.status));
+  KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch,
+             D.R, k.status, guard_args(k, st)));
   CK(cudaGetLastError());
   if (relay) {
     // Eq. 4 for every slot of every sequence; Eq. 5 keeps slots j <= n_carry
@@ -1027,20 +1081,29 @@ dflow_status do_draft(const Call &k, dflow_state *st, int *blk, int relay, float
     CK(cudaGetLastError());
     return DFLOW_OK;
   }
-  CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, logits));
-  KL(klaunch(k_draft_out, (rows + 127) / 128, 128, 0, k.s, h->gd, st->tokens, st->seq_len, h->cfg.max_ctx, batch,
-                                                   D.R, blk, k.status));
-  CK(cudaGetLastError());
+  BlockOut bo;
+  bo.blk = blk;
+  bo.tokens = st->tokens;
+  bo.seq_len = st->seq_len;
+  bo.max_ctx = h->cfg.max_ctx;
+  bo.R = D.R;
+  CK(lm_head_argmax<T>(k, D, rows, h->w.draft_final_norm, h->gd, logits, bo));
   return DFLOW_OK;
 }
 
 template <typename T>
-dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, void *feats, float *logits) {
+// rows_ready: the round's drafting already wrote pos / wr / kvlen for these rows
+// (seq_len is unchanged in between), so k_rows_round is not run again
+dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, void *feats, float *logits,
+                       bool rows_ready = false) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch, D.R, k.status));
-  CK(cudaGetLastError());
+  if (!rows_ready) {
+    KL(klaunch(k_rows_round, (rows + 127) / 128, 128, 0, k.s, h->pos, h->wr, h->kvlen, st->seq_len, st->active, batch,
+               D.R, k.status, guard_args(k, st)));
+    CK(cudaGetLastError());
+  }
   KL(klaunch(k_embed<T>, rows, 256, 0, k.s, (const T *)h->w.embed, blk, D.R, D.R, (const int *)nullptr, h->x, D.d,
              D.vocab, h->fused ? (T *)h->xn : nullptr, h->tl[0].attn_norm, h->ss, h->rows_max, k.status_w));
   CK(cudaGetLastError());
@@ -1048,23 +1111,29 @@ dflow_status do_verify(const Call &k, dflow_state *st, const int *blk, int *g, v
   return DFLOW_OK;
 }
 
+// carry_rows: also write the context rows' positions for the do_carry that follows
 dflow_status do_accept(const Call &k, dflow_state *st, const int *blk, const int *g, const int *forced,
-                       int *acc, int *comm) {
+                       int *acc, int *comm, bool carry_rows = false) {
   dflow_handle *h = k.h;
   KL(klaunch(k_accept, (st->batch + 31) / 32, 32, 0, k.s, blk, g, forced, st->tokens, st->seq_len, st->active,
-                                                 st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w));
+                                                 st->batch, h->D.B, h->cfg.max_ctx, acc, comm, k.status_w,
+                                                 carry_rows ? h->pos2 : nullptr, carry_rows ? h->wr2 : nullptr));
   CK(cudaGetLastError());
   return DFLOW_OK;
 }
 
 template <typename T>
+// rows_ready: the accept kernel of the same round already wrote pos2 / wr2
 dflow_status do_carry(const Call &k, dflow_state *st, const int *blk, const void *feats, const int *acc,
-                      int relay) {
+                      int relay, bool rows_ready = false) {
   dflow_handle *h = k.h;
   const Dims D = round_dims(h);
   const int batch = st->batch, rows = batch * D.R;
-  KL(klaunch(k_carry_rows, (rows + 127) / 128, 128, 0, k.s, acc, st->seq_len, batch, D.R, h->pos2, h->wr2, k.status));
-  CK(cudaGetLastError());
+  if (!rows_ready) {
+    KL(klaunch(k_carry_rows, (rows + 127) / 128, 128, 0, k.s, acc, st->seq_len, batch, D.R, h->pos2, h->wr2,
+               k.status));
+    CK(cudaGetLastError());
+  }
   CK(ctx_append<T>(k, D, rows, st, feats));
   KL(klaunch(k_carry<T>, dim3(batch, D.B), 256, 0, k.s, (const T *)feats, acc, blk, st->tokens, st->seq_len,
                                                h->cfg.max_ctx, (T *)st->carry, st->n_carry, st->boundary,
@@ -1083,7 +1152,7 @@ dflow_status do_round_sampled(const Call &k, dflow_state *st, SampRound sr, int 
   const int batch = st->batch, R = h->R;
   dflow_status r;
   if ((r = do_draft<T>(k, st, h->blk, relay, qlog, &sr))) return r;
-  if ((r = do_verify<T>(k, st, h->blk, nullptr, h->feats, plog))) return r;
+  if ((r = do_verify<T>(k, st, h->blk, nullptr, h->feats, plog, true))) return r;
   int n = 0;
   const cudaError_t e = samp_verify(plog, qlog, h->D.vocab, R, batch, sr, h->samp, h->blk, st->active, h->g,
                                     k.status, k.s, &n);
@@ -1091,8 +1160,8 @@ dflow_status do_round_sampled(const Call &k, dflow_state *st, SampRound sr, int 
   h->dep.brk();
   CK(e);
   CK(cudaGetLastError());
-  if ((r = do_accept(k, st, h->blk, h->g, h->samp.a, acc, comm))) return r;
-  return do_carry<T>(k, st, h->blk, h->feats, acc, relay);
+  if ((r = do_accept(k, st, h->blk, h->g, h->samp.a, acc, comm, true))) return r;
+  return do_carry<T>(k, st, h->blk, h->feats, acc, relay, true);
 }
 
 // Sec. 5.2 baseline: one greedy step of the target alone.  The step runs on the
@@ -1353,7 +1422,6 @@ dflow_status dflow_draft_block(dflow_handle *h, dflow_state *st, int32_t *block_
   if (r) return r;
   if (!block_tokens) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return finish(h, r);
   return finish(h, h->dtype == DFLOW_BF16 ? do_draft<bf16>(k, st, block_tokens, 1, logits)
                                           : do_draft<float>(k, st, block_tokens, 1, logits));
 }
@@ -1364,7 +1432,6 @@ dflow_status dflow_verify_block(dflow_handle *h, dflow_state *st, const int32_t 
   if (r) return r;
   if (!block_tokens || !target_argmax || !feats) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return finish(h, r);
   return finish(h, h->dtype == DFLOW_BF16 ? do_verify<bf16>(k, st, block_tokens, target_argmax, feats, logits)
                                           : do_verify<float>(k, st, block_tokens, target_argmax, feats, logits));
 }
@@ -1395,17 +1462,16 @@ dflow_status dflow_round(dflow_handle *h, dflow_state *st, const int32_t *forced
   if (r) return r;
   if (!accept_len || !committed) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return finish(h, r);
   if (h->dtype == DFLOW_BF16) {
     if ((r = do_draft<bf16>(k, st, h->blk, relay))) return finish(h, r);
-    if ((r = do_verify<bf16>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
-    if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
-    return finish(h, do_carry<bf16>(k, st, h->blk, h->feats, accept_len, relay));
+    if ((r = do_verify<bf16>(k, st, h->blk, h->g, h->feats, nullptr, true))) return finish(h, r);
+    if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed, true))) return finish(h, r);
+    return finish(h, do_carry<bf16>(k, st, h->blk, h->feats, accept_len, relay, true));
   }
   if ((r = do_draft<float>(k, st, h->blk, relay))) return finish(h, r);
-  if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr))) return finish(h, r);
-  if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed))) return finish(h, r);
-  return finish(h, do_carry<float>(k, st, h->blk, h->feats, accept_len, relay));
+  if ((r = do_verify<float>(k, st, h->blk, h->g, h->feats, nullptr, true))) return finish(h, r);
+  if ((r = do_accept(k, st, h->blk, h->g, forced_accept, accept_len, committed, true))) return finish(h, r);
+  return finish(h, do_carry<float>(k, st, h->blk, h->feats, accept_len, relay, true));
 }
 
 dflow_status dflow_round_sampled(dflow_handle *h, dflow_state *st, uint64_t seed, int32_t round_index,
@@ -1415,7 +1481,6 @@ dflow_status dflow_round_sampled(dflow_handle *h, dflow_state *st, uint64_t seed
   if (r) return r;
   if (!accept_len || !committed || round_index < 0 || round_index >= (1 << 24)) return DFLOW_ERR_INVALID_ARG;
   Call k = make_call(h, st, stream);
-  if ((r = guard(k, st))) return finish(h, r);
   const SampRound sr{seed, round_index};
   float *q = draft_logits ? draft_logits : h->qlog, *p = verify_logits ? verify_logits : h->plog;
   return finish(h, h->dtype == DFLOW_BF16 ? do_round_sampled<bf16>(k, st, sr, accept_len, committed, relay, q, p)
@@ -1500,7 +1565,8 @@ dflow_status dflow_debug_gemm(dflow_handle *h, int32_t path, const void *W, int3
   if (e == cudaErrorNotSupported) return DFLOW_ERR_UNSUPPORTED;
   CK(e);
   if (mode == EP_ARGMAX) {
-    klaunch(k_argmax_reduce, (M + 7) / 8, 256, 0, s, h->am_val, h->am_idx, ep.n_tiles, M, static_cast<int *>(out), status);
+    klaunch(k_argmax_reduce, (M + 7) / 8, 256, 0, s, h->am_val, h->am_idx, ep.n_tiles, M, static_cast<int *>(out), status,
+            BlockOut{});
     CK(cudaGetLastError());
   }
   return DFLOW_OK;

@@ -127,13 +127,6 @@ cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const
   const long long units = (long long)D.hkv * batch * ((D.R * G + T5_ROWS - 1) / T5_ROWS);
   const int r8 = t5_resident_clusters<BLOCK, 8>(smem), r4 = t5_resident_clusters<BLOCK, 4>(smem);
   if (r8 < 1) return cudaErrorInvalidValue;
-  // DFLOW_ATTN_SPLITS=4 or 8 fixes the cluster size (for timing the choice)
-  static const int forced = [] {
-    const char *e = getenv("DFLOW_ATTN_SPLITS");
-    return e ? atoi(e) : 0;
-  }();
-  if (forced == 4 && r4 >= 1) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
-  if (forced == 8) return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
   // 8 splits only when every cluster is resident at once; otherwise 4 (fewer,
   // longer CTAs: at batch 16 and 1K-8K keys a launch took 0.64-0.70 of the time)
   if (units > r8) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
