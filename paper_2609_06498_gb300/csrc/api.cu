@@ -83,22 +83,29 @@ __global__ void k_rows_round(int *pos, int *wr, int *kvlen, const int *seq_len, 
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= batch * R) return;
   const int b = r / R, i = r % R;
-  if (gd.status != nullptr && i == 0 && active[b]) {
+  bool ok = active[b] != 0;
+  if (gd.status != nullptr && ok) {
+    // every row of a sequence whose block would not fit gets no write (the
+    // projections that follow place K/V by these positions and do not read the
+    // status word); the block's other checks only set the status
     const int n = seq_len[b];
-    if (n < 1 || n - 1 + R > gd.max_ctx) {
-      set_status(gd.status, DFLOW_ERR_CAPACITY);
-    } else {
-      const int anchor = gd.tokens[(size_t)b * gd.max_ctx + n - 1];
-      const int nc = gd.n_carry[b];
-      if (anchor < 0 || anchor >= gd.vocab || nc < 0 || nc > gd.B - 1) {
-        set_status(gd.status, DFLOW_ERR_BAD_STATE);
-      } else if (nc > 0) {
-        const int t0 = gd.boundary[2 * b], t1 = gd.boundary[2 * b + 1];
-        if (t0 < 0 || t0 >= gd.vocab || t1 < 0 || t1 >= gd.vocab) set_status(gd.status, DFLOW_ERR_BAD_STATE);
+    const bool fits = n >= 1 && n - 1 + R <= gd.max_ctx;
+    if (i == 0) {
+      if (!fits) {
+        set_status(gd.status, DFLOW_ERR_CAPACITY);
+      } else {
+        const int anchor = gd.tokens[(size_t)b * gd.max_ctx + n - 1];
+        const int nc = gd.n_carry[b];
+        if (anchor < 0 || anchor >= gd.vocab || nc < 0 || nc > gd.B - 1) {
+          set_status(gd.status, DFLOW_ERR_BAD_STATE);
+        } else if (nc > 0) {
+          const int t0 = gd.boundary[2 * b], t1 = gd.boundary[2 * b + 1];
+          if (t0 < 0 || t0 >= gd.vocab || t1 < 0 || t1 >= gd.vocab) set_status(gd.status, DFLOW_ERR_BAD_STATE);
+        }
       }
     }
+    ok = fits;
   }
-  const bool ok = active[b] != 0;
   pos[r] = ok ? seq_len[b] - 1 + i : 0;
   wr[r] = ok;
   if (i == 0) kvlen[b] = ok ? seq_len[b] - 1 + R : 1;  // causal keys 0..n-2+R once the block is written

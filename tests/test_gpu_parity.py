@@ -253,6 +253,17 @@ def test_device_errors_are_reported(setup):
     st2.n_carry.fill_(cfg.block)
     eng.draft_block(st2)
     assert eng.read_status(st2) == 6
+    # the same checks open the T = 1 round and the verify call
+    st3 = eng.new_state(cfg.batch)
+    st3.seq_len.fill_(st3.max_ctx - 2)
+    eng.round_sampled(st3, 1, 0)
+    assert eng.read_status(st3) == 3
+    st4 = eng.new_state(cfg.batch)
+    st4.seq_len.fill_(5)
+    st4.tokens[:, 4] = cfg.vocab  # the anchor is not a token
+    blk = torch.zeros(cfg.batch, cfg.rows, dtype=torch.int32, device="cuda")
+    eng.verify_block(st4, blk)
+    assert eng.read_status(st4) == 6
 
 
 @pytest.mark.parametrize("ctx", [[3905, 4100, 2001], [64 * 41 + 1, 64 * 60, 130]])
