@@ -130,7 +130,9 @@ __device__ __forceinline__ void t5_unit(const CUtensorMap *tm, const CUtensorMap
   // page table is the caller's.  Q and the pages with the block's own rows,
   // written by the projection just before, are read after the wait.
   int pg = 0, n_pre = 0, n_early = 0;
-  const int nk = a.causal ? a.kvlen[b] : a.seq_len[b] - 1;
+  // keys of the sequence, never past its page-table row (a state that fails the
+  // round's checks sets the status, but every CTA of a cluster still runs the unit)
+  const int nk = min(a.causal ? a.kvlen[b] : a.seq_len[b] - 1, D.pages_per_seq * 64);
   auto issue_page = [&](int it, int page) {  // warp 0, lane 0: page tile `page` into stage it
     uint8_t *kt = ring + (size_t)it * 2 * TILE, *vt = kt + TILE;
     const int rk = ((page * 2 + 0) * D.hkv + kvh) * 64, rv = ((page * 2 + 1) * D.hkv + kvh) * 64;

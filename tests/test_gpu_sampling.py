@@ -164,6 +164,34 @@ def test_sampled_round_is_deterministic_and_seeded(setup):
     assert not np.array_equal(outs[0][1], outs[2][1])
 
 
+def test_sampled_round_leaves_inactive_sequences_untouched(setup):
+    """A frozen sequence (active = 0) keeps its tokens, length, carry and boundary
+    and reports accept_len -1; the others still follow the oracle's rule."""
+    cfg, o, eng = setup
+    if cfg.batch < 2:
+        pytest.skip("needs two sequences")
+    R, V, bs = cfg.rows, cfg.vocab, cfg.batch
+    ost = _start_state(cfg, o)
+    ost.active[1] = False
+    st = eng.new_state(bs, page_seed=4)
+    upload_state(eng, st, ost)
+    before = {k: to_np(getattr(st, k)).copy() for k in ("tokens", "seq_len", "n_carry", "boundary")}
+    carry0 = to_np(st.carry)[1].copy()
+    QL = torch.zeros(bs, R, V, device="cuda")
+    PL = torch.zeros(bs, R, V, device="cuda")
+    acc, comm = eng.round_sampled(st, SEED, 2, logits=(QL, PL))
+    assert eng.read_status(st) == 0
+    ga, gc, gb = to_np(acc), to_np(comm), to_np(st.boundary)
+    assert ga[1] == -1 and (gc[1] == -1).all()
+    for k, v in before.items():
+        assert np.array_equal(to_np(getattr(st, k))[1], v[1]), k
+    assert np.array_equal(to_np(st.carry)[1], carry0)
+    ql, pl = to_np(QL), to_np(PL)
+    for b in (0, 2):
+        if b < bs:
+            check_own_logits(cfg, b, ql[b], pl[b], ga, gc, gb, synth.sampling_noise(cfg, b, 2, SEED))
+
+
 def test_sampled_round_rejects_bad_round_index(setup):
     from paper_2609_06498_gb300._abi import DFlowError
     cfg, o, eng = setup
