@@ -117,8 +117,11 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs 
 }
 
 // eight key splits per (kv head, sequence, query group) when every eight-CTA
-// cluster is resident at once, else four (a CTA's fixed costs, set-up, first
-// pages and the cluster merge, are paid by half as many CTAs)
+// cluster is resident at once, else four when those all are, else two: a CTA's
+// fixed costs (set-up, first pages, the cluster merge) are paid by fewer CTAs, and
+// smaller clusters leave fewer SMs of a GPC idle.  (One split per unit measured
+// faster on equal contexts but slower on ragged ones: the longest sequence's
+// CTA then sets the launch time.)
 template <bool BLOCK>
 cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
                           cudaStream_t s, DepChain *chain) {
@@ -127,10 +130,11 @@ cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const
   const long long units = (long long)D.hkv * batch * ((D.R * G + T5_ROWS - 1) / T5_ROWS);
   const int r8 = t5_resident_clusters<BLOCK, 8>(smem), r4 = t5_resident_clusters<BLOCK, 4>(smem);
   if (r8 < 1) return cudaErrorInvalidValue;
-  // 8 splits only when every cluster is resident at once; otherwise 4 (fewer,
-  // longer CTAs: at batch 16 and 1K-8K keys a launch took 0.64-0.70 of the time)
-  if (units > r8) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
-  return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
+  if (units <= r8) return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
+  if (units <= r4) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
+  // (the query also sets the 2-split kernel's shared-memory limit)
+  if (t5_resident_clusters<BLOCK, 2>(smem) < 1) return cudaErrorInvalidValue;
+  return launch_t5<BLOCK, 2>(tm, D, batch, a, status, s, chain, smem);
 }
 
 }  // namespace
