@@ -968,12 +968,14 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
       } else {
         // this CTA's partial of row r into its slot, then free the accumulator
-        float *const mine = p.slots + (((size_t)t * p.P + rank) * BM + r) * p.npad;
+        // a slot is [npad / 16 column chunks][BM rows][16]: a warp's stores of one
+        // chunk are one contiguous 2 KB run
+        float *const mine = p.slots + ((size_t)t * p.P + rank) * BM * p.npad + (size_t)r * 16;
         for (int c0 = 0; c0 < cols; c0 += 16) {
           tmem_ld16(acc_addr + c0, v);
 #pragma unroll
           for (int q4 = 0; q4 < 4; ++q4)
-            __stcg(reinterpret_cast<float4 *>(mine + c0 + 4 * q4),
+            __stcg(reinterpret_cast<float4 *>(mine + (size_t)c0 * BM + 4 * q4),
                    make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
         }
         tc_fence_before();
@@ -985,8 +987,8 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         if (leader) sm.left_last = atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(p.P - 1) ? 1 : 0;
         epi_bar();
         if (sm.left_last) {
-          const float *const row0 = p.slots + ((size_t)t * p.P * BM + r) * p.npad;
-          const size_t rstride = (size_t)BM * p.npad;
+          const float *const row0 = p.slots + (size_t)t * p.P * BM * p.npad + (size_t)r * 16;
+          const size_t rstride = (size_t)BM * p.npad;  // one rank's slot
           for (int c0 = 0; c0 < cols; c0 += 16) {
             epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
 #pragma unroll
@@ -994,7 +996,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
             for (int rr = 0; rr < p.P; ++rr) {
 #pragma unroll
               for (int q4 = 0; q4 < 4; ++q4) {
-                const float4 y = __ldcg(reinterpret_cast<const float4 *>(row0 + rr * rstride + c0 + 4 * q4));
+                const float4 y = __ldcg(reinterpret_cast<const float4 *>(row0 + rr * rstride + (size_t)c0 * BM + 4 * q4));
                 v[4 * q4] += y.x;
                 v[4 * q4 + 1] += y.y;
                 v[4 * q4 + 2] += y.z;
