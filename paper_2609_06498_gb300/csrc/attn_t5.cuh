@@ -39,6 +39,7 @@ template <int KVS>
 struct T5Bars {
   uint64_t kv_full[KVS], kv_empty[KVS], s_full[2], s_free[2], p_ready[2], pv_done[2], q_full, drain;
   int n_keys;
+  uint32_t tmem;  // the launch's TMEM columns (attention launch)
   float m[T5_ROWS], l[T5_ROWS];
 };
 // bytes of the unit's shared-memory region: Q [2][128][128 B], KVS K/V stages, 2 P tiles

@@ -18,6 +18,13 @@ using namespace ptx;
 using namespace t5;
 
 constexpr int THREADS = 192;  // warp 0 loads, warp 1 issues MMAs, warps 2-5 run the softmax
+// K/V pages in flight: five with 8- and 4-CTA clusters (a split's pages at 2K keys
+// and batch 1-4 are then all issued before the dependency wait), four with 2-CTA
+// clusters (long contexts at batch 16 measured slightly faster so)
+template <int S>
+constexpr int t5_kvs() { return S >= 4 ? 5 : 4; }
+template <int S>
+constexpr size_t t5_smem() { return 1024 + t5_region_bytes<t5_kvs<S>()>() + sizeof(T5Bars<t5_kvs<S>()>); }
 
 // ===========================================================================
 // Queries are the MMA's M (padded to 128),
@@ -40,14 +47,13 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   // runs even after an earlier error (every wait is bounded): the CTAs of a
   // cluster must not disagree on whether to take part in its barriers
   pdl_trigger();
-  constexpr int KVS = 4;
+  constexpr int KVS = t5_kvs<S>();
   extern __shared__ __align__(1024) uint8_t dsm[];
   uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(dsm) + 1023) & ~(uintptr_t)1023);
   T5Bars<KVS> &sm = *reinterpret_cast<T5Bars<KVS> *>(base + t5_region_bytes<KVS>());
-  __shared__ uint32_t tmem_slot;
   const int warp = threadIdx.x / 32;
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&sm.tmem)),
                  "r"(T5_TMEM_COLS)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
@@ -55,7 +61,7 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = tmem_slot;
+  const uint32_t tmem = sm.tmem;
   t5_unit<BLOCK, S, KVS, THREADS>(&tm, &tq, D, a, q_tma, base, sm, tmem, (int)blockIdx.x, (int)blockIdx.y,
                                   (int)blockIdx.z / S, (int)blockIdx.z % S, &a.dep, status);
   if (threadIdx.x == 0) dep_signal(a.dep);  // every global write of this CTA is done
@@ -67,7 +73,8 @@ k_attn_t5(const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtens
 
 // resident clusters of S CTAs of k_attn_t5<BLOCK, S> (0 when the query fails)
 template <bool BLOCK, int S>
-int t5_resident_clusters(size_t smem) {
+int t5_resident_clusters() {
+  constexpr size_t smem = t5_smem<S>();
   static int n = -1;
   if (n >= 0) return n;
   n = 0;
@@ -92,7 +99,8 @@ int t5_resident_clusters(size_t smem) {
 
 template <bool BLOCK, int S>
 cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs a, int *status, cudaStream_t s,
-                      DepChain *chain, size_t smem) {
+                      DepChain *chain) {
+  constexpr size_t smem = t5_smem<S>();
   const int G = D.hq / D.hkv;
   const int qgroups = (D.R * G + T5_ROWS - 1) / T5_ROWS;
   // one group of query rows: they arrive as two 3D boxes (64 dims x G heads x R rows)
@@ -125,16 +133,15 @@ cudaError_t launch_t5(const CUtensorMap &tm, const Dims &D, int batch, AttnArgs 
 template <bool BLOCK>
 cudaError_t launch_t5_any(const CUtensorMap &tm, const Dims &D, int batch, const AttnArgs &a, int *status,
                           cudaStream_t s, DepChain *chain) {
-  const size_t smem = 1024 + t5_region_bytes<4>() + sizeof(T5Bars<4>);
   const int G = D.hq / D.hkv;
   const long long units = (long long)D.hkv * batch * ((D.R * G + T5_ROWS - 1) / T5_ROWS);
-  const int r8 = t5_resident_clusters<BLOCK, 8>(smem), r4 = t5_resident_clusters<BLOCK, 4>(smem);
+  const int r8 = t5_resident_clusters<BLOCK, 8>(), r4 = t5_resident_clusters<BLOCK, 4>();
   if (r8 < 1) return cudaErrorInvalidValue;
-  if (units <= r8) return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain, smem);
-  if (units <= r4) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain, smem);
+  if (units <= r8) return launch_t5<BLOCK, 8>(tm, D, batch, a, status, s, chain);
+  if (units <= r4) return launch_t5<BLOCK, 4>(tm, D, batch, a, status, s, chain);
   // (the query also sets the 2-split kernel's shared-memory limit)
-  if (t5_resident_clusters<BLOCK, 2>(smem) < 1) return cudaErrorInvalidValue;
-  return launch_t5<BLOCK, 2>(tm, D, batch, a, status, s, chain, smem);
+  if (t5_resident_clusters<BLOCK, 2>() < 1) return cudaErrorInvalidValue;
+  return launch_t5<BLOCK, 2>(tm, D, batch, a, status, s, chain);
 }
 
 }  // namespace

@@ -109,6 +109,39 @@ def test_full_width_round_calls(full):
     assert eng.read_status(st) == 0
 
 
+def test_ragged_contexts_two_split_attention():
+    """Batch 6 x 8 kv heads is more (kv head, sequence) units than one wave of
+    4-CTA clusters holds, so both attentions run 2-CTA clusters, with contexts of
+    2 to 65 pages (partial last pages) in one launch."""
+    from paper_2609_06498_gb300 import Engine, build, pack_weights
+    build.build()
+    cfg = reduced(synth.QWEN3_8B_KV).replace(name="kv_b6_ragged", batch=6, prompt_len=70, ctx_range=(70, 4100))
+    W = synth.weights(cfg, perturb_norms=True)
+    eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
+    o = Oracle(cfg, {k: v.astype(np.float64) for k, v in W.items()})
+    lens = np.array([70, 4100, 1500, 130, 2900, 700], np.int32)
+    nc = np.array([5, 0, 15, 9, 1, 3], np.int32)
+    ost = o.state_from_synthetic(synth.synthetic_state(cfg, ctx_lens=lens, n_carry=nc))
+    R, bs = cfg.rows, cfg.batch
+    st = eng.new_state(bs, page_seed=21)
+    upload_state(eng, st, ost)
+    ref = ost.copy()
+    gblk, gdl = eng.draft_block(st, logits=True)
+    gdl = to_np(gdl)
+    oblk = np.zeros((bs, R), np.int32)
+    for b in range(bs):
+        oblk[b], lg, _ = o.draft_block(ref, b)
+        assert_close(gdl[b, 1:], lg[1:], cfg, "draft logits")
+    g, feats, logits = eng.verify_block(st, torch.as_tensor(oblk).cuda(), logits=True)
+    gl = to_np(logits)
+    for b in range(bs):
+        _, lg, _ = o.verify_block(ref, b, oblk[b])
+        assert_close(gl[b], lg, cfg, "verify logits")
+    assert eng.read_status(st) == 0
+    del eng
+    torch.cuda.empty_cache()
+
+
 @pytest.mark.parametrize("name", ["qwen3_8b_b1", "qwen3_4b_b4"])
 def test_full_width_rounds(name):
     """Three dflow_round calls in a row at full widths (2 + 1 layers) from a
