@@ -64,7 +64,9 @@ struct Smem {
   // recv: this CTA's slice of the split-K partials has arrived (armed by the CTA
   // itself, completed by its peers' bytes); rfree: every owner has consumed
   // this CTA's previous pushes (one arrival per peer)
-  uint64_t full[16], empty[16], accf[2], acce[2], recv, rfree, drain;
+  // ovf (one-pass GEMM with overlapping accumulators): the epilogue has read the
+  // columns its buffer shares with the other one
+  uint64_t full[16], empty[16], accf[2], acce[2], recv, rfree, drain, ovf;
   uint32_t tmem;
   int flag;
   int abort;
@@ -822,6 +824,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
       mbar_init(&sm.acce[b], 4);
     }
     mbar_init(&sm.drain, 1);
+    mbar_init(&sm.ovf, 4);
     sm.abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -836,6 +839,15 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
   const int n_tiles = q < p.T ? (p.T - q + p.Q - 1) / p.Q : 0;  // tiles of this CTA
+  // accumulator buffers: nbuf 1: one; 2: two side by side; 3: two that share the
+  // TMEM columns [512 - npad, npad) (npad > 256): buffer 0 at column 0, buffer 1
+  // at 512 - npad.  With 3 the epilogue reads the shared columns first and
+  // arrives on ovf, and the next tile's MMAs wait for that instead of the whole
+  // epilogue.
+  const bool ovl = p.nbuf == 3;
+  auto acc_col = [&](int buf) -> uint32_t {
+    return buf == 0 ? 0u : (uint32_t)(p.nbuf == 2 ? p.npad : 512 - p.npad);
+  };
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
@@ -892,11 +904,13 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
       uint32_t ph = 0;
       bool ok = true;
       for (int i = 0; i < n_tiles && ok; ++i) {
-        const int buf = p.nbuf == 2 ? (i & 1) : 0;
-        const uint32_t par = p.nbuf == 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
+        const int buf = p.nbuf >= 2 ? (i & 1) : 0;
+        const uint32_t par = p.nbuf >= 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
         if (!mbar_wait(&sm.acce[buf], par ^ 1)) { ok = false; break; }
+        // the previous tile's epilogue has read the columns the two buffers share
+        if (ovl && i > 0 && !mbar_wait(&sm.ovf, (uint32_t)((i - 1) & 1))) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d = tmem + buf * p.npad;
+        const uint32_t d = tmem + acc_col(buf);
         for (int k = kr0; k < kr1; ++k) {
           if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
           tc_fence_after();
@@ -940,10 +954,26 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
     const int cols = p.npad < p.M ? p.npad : p.M;
     for (int i = 0; i < n_tiles; ++i) {
       const int t = q + i * p.Q;
-      const int buf = p.nbuf == 2 ? (i & 1) : 0;
-      const uint32_t par = p.nbuf == 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
+      const int buf = p.nbuf >= 2 ? (i & 1) : 0;
+      const uint32_t par = p.nbuf >= 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
+      // 16-column chunks in the order c(0), c(1), ...: with shared columns, the
+      // chunks that hold them first (buffer 0: its last ones; buffer 1: its first),
+      // then ovf
+      const int nch = (cols + 15) / 16;
+      const int c_first = ovl && buf == 0 ? (512 - p.npad) / 16 : 0;
+      const int rot = c_first < nch ? c_first : 0;
+      const int n_shared = !ovl ? -1 : buf == 0 ? (c_first < nch ? nch - c_first : 0)
+                                                : min((2 * p.npad - 512 + 15) / 16, nch);
+      auto chunk_col = [&](int k) { return 16 * ((rot + k) % nch); };
+      auto shared_read = [&](int k) {  // after the k-th chunk in this order (k = -1: before the first)
+        if (k + 1 == n_shared) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.ovf);
+        }
+      };
       EpPre pre;
-      if (p.P == 1) epilogue_prefetch<EP>(p, sm, t, r, 0, 16, pre);
+      if (p.P == 1) epilogue_prefetch<EP>(p, sm, t, r, chunk_col(0), 16, pre);
       if (leader) sm.flag = mbar_wait(&sm.accf[buf], par) ? 1 : 0;
       __syncwarp();
       epi_bar();
@@ -955,13 +985,16 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         break;
       }
       tc_fence_after();
-      const uint32_t acc_addr = lane_addr + buf * p.npad;
+      const uint32_t acc_addr = lane_addr + acc_col(buf);
       float v[16];
+      shared_read(-1);
       if (p.P == 1) {
-        for (int c0 = 0; c0 < cols; c0 += 16) {
-          if (c0 > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
+        for (int k = 0; k < nch; ++k) {
+          const int c0 = chunk_col(k);
+          if (k > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
           tmem_ld16(acc_addr + c0, v);
           epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v, pre);
+          shared_read(k);
         }
         tc_fence_before();
         __syncwarp();
@@ -971,12 +1004,14 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         // a slot is [npad / 16 column chunks][BM rows][16]: a warp's stores of one
         // chunk are one contiguous 2 KB run
         float *const mine = p.slots + ((size_t)t * p.P + rank) * BM * p.npad + (size_t)r * 16;
-        for (int c0 = 0; c0 < cols; c0 += 16) {
+        for (int k = 0; k < nch; ++k) {
+          const int c0 = chunk_col(k);
           tmem_ld16(acc_addr + c0, v);
 #pragma unroll
           for (int q4 = 0; q4 < 4; ++q4)
             __stcg(reinterpret_cast<float4 *>(mine + (size_t)c0 * BM + 4 * q4),
                    make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
+          shared_read(k);
         }
         tc_fence_before();
         __syncwarp();
@@ -1922,9 +1957,11 @@ cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const v
     p.npad = (Mc + 15) / 16 * 16;
     p.T = (N + BM - 1) / BM;
     p.kb = K / BK;
-    p.nbuf = 2 * p.npad <= 512 ? 2 : 1;
+    // two accumulators side by side when they fit, else two that share the
+    // columns [512 - npad, npad) (up to 384 token columns), else one
+    p.nbuf = 2 * p.npad <= 512 ? 2 : p.npad <= 384 ? 3 : 1;
     int cols = 32;
-    while (cols < p.nbuf * p.npad) cols <<= 1;
+    while (cols < (p.nbuf == 3 ? 512 : p.nbuf * p.npad)) cols <<= 1;
     p.tmem_cols = cols;
     const int n1 = p.npad < 256 ? p.npad : 256;
     p.idesc1 = mma_idesc(n1);
