@@ -1016,15 +1016,42 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&sm.acce[buf]);
-        // the leader's count is a release at GPU scope after every thread's stores
-        // (through the barrier), and an acquire for the last arriver's reads
+        // The leader's count is a release at GPU scope after every thread's stores
+        // (through the barrier); its wait for all P counts an acquire for every
+        // thread's reads after the next barrier.  The P CTAs of the tile are all
+        // resident (grid <= SMs, one CTA per SM, and no later launch starts before
+        // every CTA of this one has), so the wait ends; it is bounded all the same.
         epi_bar();
-        if (leader) sm.left_last = atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(p.P - 1) ? 1 : 0;
+        if (leader) {
+          atom_add_acq_rel(p.ctr + t, 1u);
+          int ok = 1;
+          const unsigned long long t0 = gtime();
+          for (int it = 0;; ++it) {
+            unsigned int v;
+            asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.ctr + t) : "memory");
+            if (v >= (unsigned)p.P) break;
+            if ((it & 15) == 15 && gtime() - t0 > WAIT_NS) {
+              ok = 0;
+              break;
+            }
+          }
+          sm.flag = ok;
+        }
         epi_bar();
-        if (sm.left_last) {
+        if (!sm.flag) {
+          if (leader) {
+            set_status(p.status, DFLOW_ERR_DEVICE_TIMEOUT);
+            atomicExch(&sm.abort, 1);
+          }
+          break;
+        }
+        // this CTA's share of the token columns: chunks [rank nch / P, (rank + 1) nch / P)
+        {
           const float *const row0 = p.slots + (size_t)t * p.P * BM * p.npad + (size_t)r * 16;
           const size_t rstride = (size_t)BM * p.npad;  // one rank's slot
-          for (int c0 = 0; c0 < cols; c0 += 16) {
+          const int k0 = rank * nch / p.P, k1 = (rank + 1) * nch / p.P;
+          for (int k = k0; k < k1; ++k) {
+            const int c0 = 16 * k;
             epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
@@ -1040,10 +1067,14 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
             }
             epilogue_chunk<EP>(p, sm, t, r, sub, lane, c0, 16, v, pre);
           }
-          if (leader) *reinterpret_cast<volatile unsigned int *>(p.ctr + t) = 0u;
         }
+        // every CTA of the tile counts again once its reads are done; the last
+        // one leaves the count at zero for the next use
+        epi_bar();
+        if (leader && atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(2 * p.P - 1))
+          *reinterpret_cast<volatile unsigned int *>(p.ctr + t) = 0u;
       }
-      epi_bar();  // sm.flag and sm.left_last are rewritten at the next tile
+      epi_bar();  // sm.flag is rewritten at the next tile
     }
   }
 
