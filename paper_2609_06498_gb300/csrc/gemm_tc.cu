@@ -1970,7 +1970,7 @@ bool gemm_wide_suits(const TcWorkspace &w, int N, int K, int M) {
   if (K < BK || K % BK) return false;
   const int Mc = M < WIDE_MAX_NPAD ? M : WIDE_MAX_NPAD;
   const WideChoice c = choose_wide((N + BM - 1) / BM, K / BK, (Mc + 15) / 16 * 16, w.sm_count, w.wslot_bytes);
-  return c.P == 1 || K / BK >= 128;
+  return c.P >= 1;
 }
 
 cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,

@@ -44,9 +44,10 @@ cudaError_t gemm_tc(const TcWorkspace &w, const void *W, int N, int K, const voi
 // One projection over up to 512 token rows per pass in a single stream of the
 // weights (any M: passes of 512 rows), split over k in independent CTAs when
 // the tiles are too few to fill the GPU; modes as gemm_tc.
-// whether gemm_wide beats the row-tiled launches for this shape: when its
-// schedule needs no k-split, or the k range is long enough (128 k-blocks or
-// more) to pay for the split's partial tiles
+// whether gemm_wide has a schedule for this shape (above 128 rows it beats the
+// row-tiled launches on every projection shape measured, k-split or not: its
+// split's partial tiles are reduced by all CTAs of the tile, each finishing its
+// share of the token columns)
 bool gemm_wide_suits(const TcWorkspace &w, int N, int K, int M);
 cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const void *X, int M, int ldx,
                       const EpArgs &ep, int *status, cudaStream_t s, DepChain *chain = nullptr);
