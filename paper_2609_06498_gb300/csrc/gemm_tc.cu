@@ -790,13 +790,58 @@ constexpr size_t WIDE_SLOT_BYTES = (size_t)48 << 20;   // split-K partials, kept
 
 struct WideParams {
   int N, K, M, npad, T, kb, P, Q, stages, tmem_cols, nbuf;
+  int Tl, ls;               // leftover tiles and the parts each is split into (P = 1 only; Tl = 0: none)
   uint32_t idesc1, idesc2;  // MMA N = min(npad, 256), and npad - 256
   EpArgs ep;
   int *status;
   Dep dep;
-  float *slots;       // [T][P][BM][npad] partials (P > 1)
+  float *slots;       // partials of the split tiles: [T][P][BM][npad], or [Tl][ls][BM][npad] for the leftovers
   unsigned int *ctr;  // [T] arrivals per tile (zero between uses)
 };
+
+// The tiles ("items") of CTA c of the one-pass GEMM, in order.  Without
+// leftovers, CTA c = q P + rank takes tiles q, q + Q, ..., each over the k range
+// `rank` of P.  With leftovers (P = 1), CTA c takes tiles c, c + Q, ... below
+// Tf = T - Tl whole, then, for c < Tl ls, the k range c % ls of ls of leftover
+// tile Tf + c / ls: every CTA streams about the same number of k-blocks.
+struct WideItem {
+  int t, k0, k1, part, parts;
+  int slot;  // index of this part's partial slot (parts > 1)
+};
+__device__ __forceinline__ int wide_n_items(const WideParams &p, int c) {
+  if (p.Tl == 0) {
+    const int q = c / p.P;
+    return q < p.T ? (p.T - q + p.Q - 1) / p.Q : 0;
+  }
+  const int Tf = p.T - p.Tl;
+  return (c < Tf ? (Tf - c + p.Q - 1) / p.Q : 0) + (c < p.Tl * p.ls ? 1 : 0);
+}
+__device__ __forceinline__ WideItem wide_item(const WideParams &p, int c, int i) {
+  WideItem it;
+  if (p.Tl == 0) {
+    const int q = c / p.P, rank = c % p.P;
+    it.t = q + i * p.Q;
+    it.part = rank;
+    it.parts = p.P;
+    it.slot = it.t * p.P + rank;
+  } else {
+    const int Tf = p.T - p.Tl, nf = c < Tf ? (Tf - c + p.Q - 1) / p.Q : 0;
+    if (i < nf) {
+      it.t = c + i * p.Q;
+      it.part = 0;
+      it.parts = 1;
+      it.slot = 0;
+    } else {
+      it.t = Tf + c / p.ls;
+      it.part = c % p.ls;
+      it.parts = p.ls;
+      it.slot = c;
+    }
+  }
+  it.k0 = it.part * p.kb / it.parts;
+  it.k1 = (it.part + 1) * p.kb / it.parts;
+  return it;
+}
 
 template <int EP>
 __global__ void __launch_bounds__(THREADS, 1)
@@ -810,8 +855,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
   const int stage_bytes = A_BYTES + p.npad * BK * 2;
   Smem &sm = *reinterpret_cast<Smem *>(ring + (size_t)p.stages * stage_bytes);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  const int q = (int)blockIdx.x / p.P, rank = (int)blockIdx.x % p.P;
-  const int kr0 = rank * p.kb / p.P, kr1 = (rank + 1) * p.kb / p.P;
+  const int cta = (int)blockIdx.x;
   const bool two = p.npad > 256;  // a second MMA (and X box) for rows 256..npad-1
 
   if (threadIdx.x == 0) {
@@ -838,7 +882,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem;
-  const int n_tiles = q < p.T ? (p.T - q + p.Q - 1) / p.Q : 0;  // tiles of this CTA
+  const int n_tiles = wide_n_items(p, cta);  // tiles (whole or a k range) of this CTA
   // accumulator buffers: nbuf 1: one; 2: two side by side; 3: two that share the
   // TMEM columns [512 - npad, npad) (npad > 256): buffer 0 at column 0, buffer 1
   // at 512 - npad.  With 3 the epilogue reads the shared columns first and
@@ -853,27 +897,44 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       const uint64_t pw = policy_evict_first(), px = policy_evict_last();
-      const int nk = kr1 - kr0, n_units = n_tiles * nk;
       auto load_x = [&](uint8_t *a, int k, uint64_t *bar) {
         tma_load_2d(a + A_BYTES, &tmX1, k * BK, 0, bar, px);
         if (two) tma_load_2d(a + A_BYTES + 256 * 128, &tmX2, k * BK, 256, bar, px);
       };
+      // the CTA's (tile, k-block) units in order
+      int wi = 0, wk = 0;
+      WideItem cur{};
+      if (n_tiles > 0) {
+        cur = wide_item(p, cta, 0);
+        wk = cur.k0;
+      }
+      auto next_unit = [&](int &t, int &k) -> bool {
+        if (wi >= n_tiles) return false;
+        t = cur.t;
+        k = wk;
+        if (++wk >= cur.k1 && ++wi < n_tiles) {
+          cur = wide_item(p, cta, wi);
+          wk = cur.k0;
+        }
+        return true;
+      };
       int n_issued = 0;
       bool ok = true;
       // weight tiles of the first ring do not depend on the previous kernel: start them now
-      const int pre = n_units < p.stages ? n_units : p.stages;
-      for (int u = 0; u < pre; ++u) {
-        mbar_expect_tx(&sm.full[u], stage_bytes);
-        tma_load_2d(ring + (size_t)u * stage_bytes, &tmW, (kr0 + u % nk) * BK, (q + (u / nk) * p.Q) * BM, &sm.full[u], pw);
+      int pre_k[16];
+      int pre = 0, t = 0, k = 0;
+      while (pre < p.stages && next_unit(t, k)) {
+        mbar_expect_tx(&sm.full[pre], stage_bytes);
+        tma_load_2d(ring + (size_t)pre * stage_bytes, &tmW, k * BK, t * BM, &sm.full[pre], pw);
+        pre_k[pre++] = k;
       }
       n_issued = pre;
       dep_wait(p.dep, p.status);
       if (p.dep.wait) fence_proxy_async_global();
-      for (int u = 0; u < pre; ++u) load_x(ring + (size_t)u * stage_bytes, kr0 + u % nk, &sm.full[u]);
+      for (int u = 0; u < pre; ++u) load_x(ring + (size_t)u * stage_bytes, pre_k[u], &sm.full[u]);
       int stage = pre % p.stages;
       uint32_t ph = pre == p.stages ? 1 : 0;
-      for (int u = pre; u < n_units; ++u) {
-        const int t = q + (u / nk) * p.Q, k = kr0 + u % nk;
+      for (int u = pre; next_unit(t, k); ++u) {
         if (!mbar_wait(&sm.empty[stage], ph ^ 1) || *(volatile int *)&sm.abort) {
           ok = false;
           break;
@@ -911,7 +972,9 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         if (ovl && i > 0 && !mbar_wait(&sm.ovf, (uint32_t)((i - 1) & 1))) { ok = false; break; }
         tc_fence_after();
         const uint32_t d = tmem + acc_col(buf);
-        for (int k = kr0; k < kr1; ++k) {
+        const WideItem it = wide_item(p, cta, i);
+        const int kr0 = it.k0;
+        for (int k = it.k0; k < it.k1; ++k) {
           if (!mbar_wait(&sm.full[stage], ph) || *(volatile int *)&sm.abort) { ok = false; break; }
           tc_fence_after();
           const uint32_t a = smem_u32(ring + (size_t)stage * stage_bytes);
@@ -953,7 +1016,8 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
     }
     const int cols = p.npad < p.M ? p.npad : p.M;
     for (int i = 0; i < n_tiles; ++i) {
-      const int t = q + i * p.Q;
+      const WideItem it = wide_item(p, cta, i);
+      const int t = it.t, rank = it.part, P = it.parts;
       const int buf = p.nbuf >= 2 ? (i & 1) : 0;
       const uint32_t par = p.nbuf >= 2 ? (uint32_t)((i >> 1) & 1) : (uint32_t)(i & 1);
       // 16-column chunks in the order c(0), c(1), ...: with shared columns, the
@@ -973,7 +1037,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         }
       };
       EpPre pre;
-      if (p.P == 1) epilogue_prefetch<EP>(p, sm, t, r, chunk_col(0), 16, pre);
+      if (P == 1) epilogue_prefetch<EP>(p, sm, t, r, chunk_col(0), 16, pre);
       if (leader) sm.flag = mbar_wait(&sm.accf[buf], par) ? 1 : 0;
       __syncwarp();
       epi_bar();
@@ -988,7 +1052,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
       const uint32_t acc_addr = lane_addr + acc_col(buf);
       float v[16];
       shared_read(-1);
-      if (p.P == 1) {
+      if (P == 1) {
         for (int k = 0; k < nch; ++k) {
           const int c0 = chunk_col(k);
           if (k > 0) epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
@@ -1003,7 +1067,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         // this CTA's partial of row r into its slot, then free the accumulator
         // a slot is [npad / 16 column chunks][BM rows][16]: a warp's stores of one
         // chunk are one contiguous 2 KB run
-        float *const mine = p.slots + ((size_t)t * p.P + rank) * BM * p.npad + (size_t)r * 16;
+        float *const mine = p.slots + (size_t)it.slot * BM * p.npad + (size_t)r * 16;
         for (int k = 0; k < nch; ++k) {
           const int c0 = chunk_col(k);
           tmem_ld16(acc_addr + c0, v);
@@ -1029,7 +1093,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
           for (int it = 0;; ++it) {
             unsigned int v;
             asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.ctr + t) : "memory");
-            if (v >= (unsigned)p.P) break;
+            if (v >= (unsigned)P) break;
             if ((it & 15) == 15 && gtime() - t0 > WAIT_NS) {
               ok = 0;
               break;
@@ -1047,15 +1111,15 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         }
         // this CTA's share of the token columns: chunks [rank nch / P, (rank + 1) nch / P)
         {
-          const float *const row0 = p.slots + (size_t)t * p.P * BM * p.npad + (size_t)r * 16;
+          const float *const row0 = p.slots + (size_t)(it.slot - rank) * BM * p.npad + (size_t)r * 16;
           const size_t rstride = (size_t)BM * p.npad;  // one rank's slot
-          const int k0 = rank * nch / p.P, k1 = (rank + 1) * nch / p.P;
+          const int k0 = rank * nch / P, k1 = (rank + 1) * nch / P;
           for (int k = k0; k < k1; ++k) {
             const int c0 = 16 * k;
             epilogue_prefetch<EP>(p, sm, t, r, c0, 16, pre);
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
-            for (int rr = 0; rr < p.P; ++rr) {
+            for (int rr = 0; rr < P; ++rr) {
 #pragma unroll
               for (int q4 = 0; q4 < 4; ++q4) {
                 const float4 y = __ldcg(reinterpret_cast<const float4 *>(row0 + rr * rstride + (size_t)c0 * BM + 4 * q4));
@@ -1071,7 +1135,7 @@ k_gemm_wide(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUt
         // every CTA of the tile counts again once its reads are done; the last
         // one leaves the count at zero for the next use
         epi_bar();
-        if (leader && atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(2 * p.P - 1))
+        if (leader && atom_add_acq_rel(p.ctr + t, 1u) == (unsigned)(2 * P - 1))
           *reinterpret_cast<volatile unsigned int *>(p.ctr + t) = 0u;
       }
       epi_bar();  // sm.flag is rewritten at the next tile
@@ -2005,6 +2069,20 @@ cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const v
     p.stages = c.stages;
     p.slots = w.wslots;
     p.ctr = w.wctr;
+    // one tile per CTA leaves T mod Q tiles over: split each over ls = Q / (T mod Q)
+    // CTAs in k (at least two k-blocks a part), so that every CTA streams about the
+    // same share instead of some CTAs a whole second tile.  Measured on gate/up
+    // (192 tiles on 152 CTAs): 79.9 against 87.1 us at 272 rows, but 88.8 against
+    // 82.7 us at 200 rows, so only above 256 token columns.
+    p.Tl = 0;
+    p.ls = 1;
+    if (p.P == 1 && p.T > p.Q && p.npad > 256) {
+      const int tl = p.T % p.Q, ls = tl > 0 ? p.Q / tl : 0;
+      if (ls >= 2 && p.kb / ls >= 2 && (size_t)tl * ls * BM * p.npad * sizeof(float) <= w.wslot_bytes) {
+        p.Tl = tl;
+        p.ls = ls;
+      }
+    }
     EpArgs ep = ep_in;
     if (ep.out_f32) ep.out_f32 += (size_t)m0 * ep.ldo;
     if (ep.out_t) ep.out_t = static_cast<bf16 *>(ep.out_t) + (size_t)m0 * ep.ldt;
