@@ -313,6 +313,23 @@ dflow_status dflow_greedy_tokens_noalloc(const void *lm_head, int32_t vocab, int
  * DFLOW_ERR_UNSUPPORTED when M or K is outside what the launch covers. */
 dflow_status dflow_debug_seq_schedule(int32_t N, int32_t K, int32_t M, int32_t Q, int32_t *plan, int32_t *ctas);
 
+/* Test hook, host only (no GPU needed): the schedule the one-pass tcgen05
+ * launch (projections above 128 rows) gives N x K weights over M <= 512 rows on
+ * `sms` SMs with `slot_bytes` of split-K partial slots, computed by the functions
+ * the launch and the kernel evaluate.
+ *   plan   int32 [10]: padded columns, tiles T, k-blocks kb, k-split P, tile
+ *          groups Q, leftover tiles Tl, parts per leftover tile ls, grid (CTAs,
+ *          P Q), accumulator buffers (1; 2 side by side; 3 sharing columns),
+ *          ring stages
+ *   items  int32 [grid][1 + 6 max_items], per CTA: its item count, then per item
+ *          (in the order it runs them) tile, k-block range [k0, k1), part, parts
+ *          (1: whole tile; more: the tile is reduced by that many CTAs, each
+ *          finishing 1/parts of the token columns), partial slot index.
+ * DFLOW_ERR_UNSUPPORTED when no schedule fits; DFLOW_ERR_CAPACITY when a CTA has
+ * more than max_items items. */
+dflow_status dflow_debug_wide_schedule(int32_t N, int32_t K, int32_t M, int32_t sms, int64_t slot_bytes,
+                                       int32_t *plan, int32_t *items, int32_t max_items);
+
 /* Waits for the recorded events, then fills out[DFLOW_PROF_N]. */
 dflow_status dflow_profile_read(dflow_handle *h, dflow_kernel_profile *out);
 /* Kernels launched by this handle since creation (always counted). */

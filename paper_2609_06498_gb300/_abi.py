@@ -76,6 +76,8 @@ _SIGS = {
     "dflow_greedy_tokens_noalloc": ([_P, ctypes.c_int32, ctypes.c_int32, _P, ctypes.c_int32, _P, _P], ctypes.c_int),
     "dflow_debug_seq_schedule": ([ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, c_i32p, c_i32p],
                                  ctypes.c_int),
+    "dflow_debug_wide_schedule": ([ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                                   c_i32p, c_i32p, ctypes.c_int32], ctypes.c_int),
     "dflow_debug_gemm": ([_P, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int32, _P, ctypes.c_int32, ctypes.c_int32,
                           ctypes.c_int32, _P, ctypes.c_int32, _P, _P], ctypes.c_int),
 }

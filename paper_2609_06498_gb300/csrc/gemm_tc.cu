@@ -808,7 +808,7 @@ struct WideItem {
   int t, k0, k1, part, parts;
   int slot;  // index of this part's partial slot (parts > 1)
 };
-__device__ __forceinline__ int wide_n_items(const WideParams &p, int c) {
+__host__ __device__ __forceinline__ int wide_n_items(const WideParams &p, int c) {
   if (p.Tl == 0) {
     const int q = c / p.P;
     return q < p.T ? (p.T - q + p.Q - 1) / p.Q : 0;
@@ -816,7 +816,7 @@ __device__ __forceinline__ int wide_n_items(const WideParams &p, int c) {
   const int Tf = p.T - p.Tl;
   return (c < Tf ? (Tf - c + p.Q - 1) / p.Q : 0) + (c < p.Tl * p.ls ? 1 : 0);
 }
-__device__ __forceinline__ WideItem wide_item(const WideParams &p, int c, int i) {
+__host__ __device__ __forceinline__ WideItem wide_item(const WideParams &p, int c, int i) {
   WideItem it;
   if (p.Tl == 0) {
     const int q = c / p.P, rank = c % p.P;
@@ -2028,6 +2028,44 @@ cudaError_t launch_wide(const CUtensorMap &mw, const CUtensorMap &mx1, const CUt
   return cudaLaunchKernelEx(&cfg, k_gemm_wide<EP>, mw, mx1, mx2, p);
 }
 
+// The one-pass launch's schedule for Mc <= WIDE_MAX_NPAD rows: padded columns,
+// accumulators, k-split and grid (choose_wide), and the leftover split; false when
+// no schedule fits.  Evaluated by the launch and by the schedule test hook.
+bool wide_plan(WideParams &p, int N, int K, int Mc, int sms, size_t slot_bytes) {
+  p.N = N;
+  p.K = K;
+  p.M = Mc;
+  p.npad = (Mc + 15) / 16 * 16;
+  p.T = (N + BM - 1) / BM;
+  p.kb = K / BK;
+  // two accumulators side by side when they fit, else two that share the
+  // columns [512 - npad, npad) (up to 384 token columns), else one
+  p.nbuf = 2 * p.npad <= 512 ? 2 : p.npad <= 384 ? 3 : 1;
+  int cols = 32;
+  while (cols < (p.nbuf == 3 ? 512 : p.nbuf * p.npad)) cols <<= 1;
+  p.tmem_cols = cols;
+  const WideChoice c = choose_wide(p.T, p.kb, p.npad, sms, slot_bytes);
+  if (c.P == 0) return false;
+  p.P = c.P;
+  p.Q = c.Q;
+  p.stages = c.stages;
+  // one tile per CTA leaves T mod Q tiles over: split each over ls = Q / (T mod Q)
+  // CTAs in k (at least two k-blocks a part), so that every CTA streams about the
+  // same share instead of some CTAs a whole second tile.  Measured on gate/up
+  // (192 tiles on 152 CTAs): 79.9 against 87.1 us at 272 rows, but 88.8 against
+  // 82.7 us at 200 rows, so only above 256 token columns.
+  p.Tl = 0;
+  p.ls = 1;
+  if (p.P == 1 && p.T > p.Q && p.npad > 256) {
+    const int tl = p.T % p.Q, ls = tl > 0 ? p.Q / tl : 0;
+    if (ls >= 2 && p.kb / ls >= 2 && (size_t)tl * ls * BM * p.npad * sizeof(float) <= slot_bytes) {
+      p.Tl = tl;
+      p.ls = ls;
+    }
+  }
+  return true;
+}
+
 }  // namespace
 
 bool gemm_wide_suits(const TcWorkspace &w, int N, int K, int M) {
@@ -2046,43 +2084,13 @@ cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const v
   for (int m0 = 0; m0 < M; m0 += WIDE_MAX_NPAD) {
     const int Mc = M - m0 < WIDE_MAX_NPAD ? M - m0 : WIDE_MAX_NPAD;
     WideParams p{};
-    p.N = N;
-    p.K = K;
-    p.M = Mc;
-    p.npad = (Mc + 15) / 16 * 16;
-    p.T = (N + BM - 1) / BM;
-    p.kb = K / BK;
-    // two accumulators side by side when they fit, else two that share the
-    // columns [512 - npad, npad) (up to 384 token columns), else one
-    p.nbuf = 2 * p.npad <= 512 ? 2 : p.npad <= 384 ? 3 : 1;
-    int cols = 32;
-    while (cols < (p.nbuf == 3 ? 512 : p.nbuf * p.npad)) cols <<= 1;
-    p.tmem_cols = cols;
+    if (!wide_plan(p, N, K, Mc, w.sm_count, w.wslot_bytes)) return cudaErrorInvalidValue;
     const int n1 = p.npad < 256 ? p.npad : 256;
     p.idesc1 = mma_idesc(n1);
     p.idesc2 = p.npad > 256 ? mma_idesc(p.npad - 256) : 0u;
     p.status = status;
-    const WideChoice c = choose_wide(p.T, p.kb, p.npad, w.sm_count, w.wslot_bytes);
-    if (c.P == 0) return cudaErrorInvalidValue;
-    p.P = c.P;
-    p.Q = c.Q;
-    p.stages = c.stages;
     p.slots = w.wslots;
     p.ctr = w.wctr;
-    // one tile per CTA leaves T mod Q tiles over: split each over ls = Q / (T mod Q)
-    // CTAs in k (at least two k-blocks a part), so that every CTA streams about the
-    // same share instead of some CTAs a whole second tile.  Measured on gate/up
-    // (192 tiles on 152 CTAs): 79.9 against 87.1 us at 272 rows, but 88.8 against
-    // 82.7 us at 200 rows, so only above 256 token columns.
-    p.Tl = 0;
-    p.ls = 1;
-    if (p.P == 1 && p.T > p.Q && p.npad > 256) {
-      const int tl = p.T % p.Q, ls = tl > 0 ? p.Q / tl : 0;
-      if (ls >= 2 && p.kb / ls >= 2 && (size_t)tl * ls * BM * p.npad * sizeof(float) <= w.wslot_bytes) {
-        p.Tl = tl;
-        p.ls = ls;
-      }
-    }
     EpArgs ep = ep_in;
     if (ep.out_f32) ep.out_f32 += (size_t)m0 * ep.ldo;
     if (ep.out_t) ep.out_t = static_cast<bf16 *>(ep.out_t) + (size_t)m0 * ep.ldt;
@@ -2105,14 +2113,15 @@ cudaError_t gemm_wide(const TcWorkspace &w, const void *W, int N, int K, const v
       mx2 = mx1;
     }
     p.dep = chain ? chain->take((unsigned)(p.P * p.Q)) : Dep{};
+    const size_t smem = 1024 + (size_t)p.stages * (A_BYTES + p.npad * BK * 2) + sizeof(Smem);  // as choose_wide
     cudaError_t e;
     switch (ep.mode) {
-      case EP_STORE_F32: e = launch_wide<EP_STORE_F32>(mw, mx1, mx2, p, c.smem, s); break;
-      case EP_RESID: e = launch_wide<EP_RESID>(mw, mx1, mx2, p, c.smem, s); break;
-      case EP_SWIGLU: e = launch_wide<EP_SWIGLU>(mw, mx1, mx2, p, c.smem, s); break;
-      case EP_SILU: e = launch_wide<EP_SILU>(mw, mx1, mx2, p, c.smem, s); break;
-      case EP_ARGMAX: e = launch_wide<EP_ARGMAX>(mw, mx1, mx2, p, c.smem, s); break;
-      case EP_QKV: e = launch_wide<EP_QKV>(mw, mx1, mx2, p, c.smem, s); break;
+      case EP_STORE_F32: e = launch_wide<EP_STORE_F32>(mw, mx1, mx2, p, smem, s); break;
+      case EP_RESID: e = launch_wide<EP_RESID>(mw, mx1, mx2, p, smem, s); break;
+      case EP_SWIGLU: e = launch_wide<EP_SWIGLU>(mw, mx1, mx2, p, smem, s); break;
+      case EP_SILU: e = launch_wide<EP_SILU>(mw, mx1, mx2, p, smem, s); break;
+      case EP_ARGMAX: e = launch_wide<EP_ARGMAX>(mw, mx1, mx2, p, smem, s); break;
+      case EP_QKV: e = launch_wide<EP_QKV>(mw, mx1, mx2, p, smem, s); break;
       default: e = cudaErrorInvalidValue;
     }
     if (e != cudaSuccess) return e;
@@ -2279,6 +2288,34 @@ cudaError_t gemm_seq(const TcWorkspace &w, int n, const SeqSpec *sp, int M, int 
 }
 
 }  // namespace dflow
+
+// Test hook (see include/dflow.h): the one-pass launch's schedule for M <= 512
+// rows, computed by the functions the launch and the kernel evaluate.
+extern "C" dflow_status dflow_debug_wide_schedule(int32_t N, int32_t K, int32_t M, int32_t sms, int64_t slot_bytes,
+                                                  int32_t *plan, int32_t *items, int32_t max_items) {
+  using namespace dflow;
+  if (N < 1 || K < BK || K % BK || M < 1 || M > WIDE_MAX_NPAD || sms < 1 || sms > 1024 || slot_bytes < 0 || !plan ||
+      !items || max_items < 1)
+    return DFLOW_ERR_INVALID_ARG;
+  WideParams p{};
+  if (!wide_plan(p, N, K, M, sms, (size_t)slot_bytes)) return DFLOW_ERR_UNSUPPORTED;
+  const int grid = p.P * p.Q;
+  const int32_t pl[10] = {p.npad, p.T, p.kb, p.P, p.Q, p.Tl, p.ls, grid, p.nbuf, p.stages};
+  for (int i = 0; i < 10; ++i) plan[i] = pl[i];
+  const size_t row = 1 + 6 * (size_t)max_items;
+  for (int c = 0; c < grid; ++c) {
+    const int n = wide_n_items(p, c);
+    if (n > max_items) return DFLOW_ERR_CAPACITY;
+    int32_t *out = items + (size_t)c * row;
+    out[0] = n;
+    for (int i = 0; i < n; ++i) {
+      const WideItem it = wide_item(p, c, i);
+      const int32_t v[6] = {it.t, it.k0, it.k1, it.part, it.parts, it.slot};
+      for (int j = 0; j < 6; ++j) out[1 + 6 * i + j] = v[j];
+    }
+  }
+  return DFLOW_OK;
+}
 
 // Test hook (see include/dflow.h): the persistent launch's schedule of one GEMM
 // over Q clusters, computed by the same functions the kernel runs.
