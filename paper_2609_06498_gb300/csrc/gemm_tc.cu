@@ -777,12 +777,15 @@ k_gemm_tc(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUten
 // ===========================================================================
 // Wide weight-streaming GEMM: up to 512 token rows in one pass over the weights
 // (two MMAs per k-step once the padded rows exceed one MMA's N of 256), for the
-// blocks of large batches.  The grid is Q tile groups x P k-splits of
-// independent CTAs: CTA (q, r) takes tiles q, q + Q, ... over k-blocks
-// [r kb / P, (r + 1) kb / P).  With P > 1 each CTA stores its fp32 partial of
-// a tile in an L2 slot; the CTA whose arrival completes the tile's count adds
-// the P slots in rank order (so the result does not depend on the arrival
-// order), runs the fused epilogue and leaves the count at zero.
+// blocks of large batches.  The grid is Q tile groups x P k-splits of CTAs:
+// CTA (q, r) takes tiles q, q + Q, ... over k-blocks [r kb / P, (r + 1) kb / P)
+// (or, with leftovers, whole tiles and then one k part of a leftover tile; see
+// wide_item).  A tile split over several CTAs is reduced by all of them: each
+// stores its fp32 partial in an L2 slot and counts it, waits until the tile's
+// parts are all in (the grid is at most one CTA per SM, so they are resident
+// together), adds the slots in part order (so the result does not depend on the
+// arrival order) for its share of the token columns and runs the fused epilogue
+// on them; a second count lets the last one leave the counter at zero.
 // ===========================================================================
 constexpr int WIDE_MAX_NPAD = 512;
 constexpr int WIDE_MAX_TILES = 4096;                    // 128-row tiles of one projection (N <= 524288)
@@ -1978,8 +1981,10 @@ struct WideChoice {
 };
 
 // k-splits and tile groups minimising the k-blocks each CTA streams, with a
-// charge for writing a split tile's partial to L2 and for the last arriver
-// reading the P partials back (both in k-block equivalents at L2 speed)
+// charge for writing a split tile's partial to L2 and reading partials back
+// (in k-block equivalents at L2 speed); the charge was set when one CTA read all
+// P partials back, and its choices still match the fastest measured P on the
+// batch-16 projections (O 4, QKV 3, down 4)
 WideChoice choose_wide(int T, int kb, int npad, int sms, size_t slot_bytes) {
   WideChoice best;
   const int stage_bytes = A_BYTES + npad * BK * 2;
