@@ -109,18 +109,21 @@ def test_full_width_round_calls(full):
     assert eng.read_status(st) == 0
 
 
-def test_ragged_contexts_two_split_attention():
-    """Batch 6 x 8 kv heads is more (kv head, sequence) units than one wave of
+@pytest.mark.parametrize("bs", [6, 9])
+def test_ragged_contexts_two_split_attention(bs):
+    """Batch 6 or 9 x 8 kv heads is more (kv head, sequence) units than one wave of
     4-CTA clusters holds, so both attentions run 2-CTA clusters, with contexts of
-    2 to 65 pages (partial last pages) in one launch."""
+    2 to 65 pages (partial last pages) in one launch.  At batch 9 the 153 rows also
+    take the one-pass GEMM (above 128 rows): k-split projections reduced by every CTA
+    of a tile, the Q/K/V epilogue included."""
     from paper_2609_06498_gb300 import Engine, build, pack_weights
     build.build()
-    cfg = reduced(synth.QWEN3_8B_KV).replace(name="kv_b6_ragged", batch=6, prompt_len=70, ctx_range=(70, 4100))
+    cfg = reduced(synth.QWEN3_8B_KV).replace(name=f"kv_b{bs}_ragged", batch=bs, prompt_len=70, ctx_range=(70, 4100))
     W = synth.weights(cfg, perturb_norms=True)
     eng = Engine(cfg, pack_weights(cfg, W), max_batch=cfg.batch, max_ctx=cfg.max_ctx())
     o = Oracle(cfg, {k: v.astype(np.float64) for k, v in W.items()})
-    lens = np.array([70, 4100, 1500, 130, 2900, 700], np.int32)
-    nc = np.array([5, 0, 15, 9, 1, 3], np.int32)
+    lens = np.array([70, 4100, 1500, 130, 2900, 700, 2049, 64 * 17 + 5, 3333], np.int32)[:bs]
+    nc = np.array([5, 0, 15, 9, 1, 3, 7, 12, 2], np.int32)[:bs]
     ost = o.state_from_synthetic(synth.synthetic_state(cfg, ctx_lens=lens, n_carry=nc))
     R, bs = cfg.rows, cfg.batch
     st = eng.new_state(bs, page_seed=21)
